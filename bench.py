@@ -1,0 +1,400 @@
+#!/usr/bin/env python3
+"""SkewAdam optimizer-step benchmark on GB300.
+
+A step is one SkewAdam update (all tiers: factored second moments, backbone
+momentum, exact router / vector second moments, update-RMS clipping, decoupled
+weight decay, dithered bf16 write-back) over a synthetic parameter set shaped
+like the paper's 6.78B-parameter MoE (App. B shapes: 6,784,327,680 bf16
+parameters in 408 tensors). Weights ~ N(0, 0.02^2), gradients ~ N(0, 1e-3^2),
+resident in HBM; 27.1 GB of weights + gradients per step is far larger than the
+129 MiB L2, so no flush is needed between steps.
+
+Reported (one JSON line, rank 0):
+  value       -- parameters updated per second, whole job (all ranks);
+  ms_per_step -- device time per step (CUDA events, max over ranks);
+  hbm         -- algorithmic minimum bytes per step / step time, and its share
+                 of the 8 TB/s nominal and of the measured copy bandwidth;
+  roofline    -- the dominant kernel's algorithmic bytes / its event-timed
+                 duration against the measured HBM copy peak;
+  e2e         -- the same metric through the C ABI with the gradients copied
+                 in from pinned host memory and the weights read back each step;
+  cpu_baseline-- the CPU oracle (single thread) on a bounded sample.
+Multi-GPU (torchrun): every rank updates its own full parameter set (the step
+has no cross-tensor coupling, so it shards by tensor with no collective);
+scaling is weak.
+
+--impl reference times the CPU oracle (the reference arm of this benchmark) on
+the host cores instead, on bounded samples of the same workload.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="appb", help="shape set (appb = the paper's 6.78B App. B shapes)")
+    p.add_argument("--seed", type=int, default=20260207)
+    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0, help="target oracle time of the CPU baseline sample")
+    p.add_argument("--ref-seconds", type=float, default=150.0, help="target total time of --impl reference")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(path))
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# nvidia-smi clock sampling during the timed region
+# ---------------------------------------------------------------------------
+CLOCK_Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+           "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+           "clocks_event_reasons.sw_power_cap")
+
+
+def clocks_start(dev_index):
+    f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+    try:
+        p = subprocess.Popen(["nvidia-smi", f"--query-gpu={CLOCK_Q}", "--format=csv,noheader,nounits", "-lms", "100",
+                              "-i", str(dev_index)], stdout=f, stderr=subprocess.DEVNULL)
+    except Exception:
+        p = None
+    return p, f
+
+
+def clocks_stop(handle):
+    p, f = handle
+    if p is None:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+    p.terminate()
+    try:
+        p.wait(timeout=5)
+    except Exception:
+        p.kill()
+    f.seek(0)
+    sm, smax, reasons, pw = [], [], set(), []
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for line in f.read().splitlines():
+        c = [x.strip() for x in line.split(",")]
+        if len(c) < 9:
+            continue
+        try:
+            sm.append(float(c[1]))
+            smax.append(float(c[2]))
+            pw.append(float(c[3]))
+        except ValueError:
+            continue
+        for n, v in zip(names, c[5:9]):
+            if v.lower().startswith("active"):
+                reasons.add(n)
+    os.unlink(f.name)
+    return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+            "reasons": sorted(reasons), "samples": len(sm), "power_w_max": max(pw) if pw else None}
+
+
+# ---------------------------------------------------------------------------
+# byte accounting
+# ---------------------------------------------------------------------------
+def byte_model(opt, n_tensors):
+    """Algorithmic minimum bytes of one step and of each kernel's own traffic."""
+    N = N_mom = N_full = N_fact = N_nomom = 0
+    rc = 0
+    for k in range(n_tensors):
+        i = opt.info(k)
+        N += i.numel
+        if i.momentum:
+            N_mom += i.numel
+        else:
+            N_nomom += i.numel
+        if i.kind == 0:
+            N_full += i.numel
+        else:
+            N_fact += i.numel
+            rc += i.rows + i.cols
+    step_min = 6 * N + 8 * N_mom + 8 * N_full + 8 * rc
+    kernels = {
+        "k_sumsq": 2 * N_fact,                                   # read G of factored matrices
+        "k_finalize": 8 * rc,                                    # R, C read + write
+        "k_rms": 2 * N + 8 * N_mom + 8 * N_full,                 # read G; M, v read + write
+        "k_apply": 4 * N + 2 * N_nomom + 4 * N_mom + 4 * N_full,  # W r/w; G or M; v read
+    }
+    return dict(N=N, N_mom=N_mom, N_full=N_full, rc=rc, step_min=step_min, kernels=kernels)
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (reported baseline / reference arm)
+# ---------------------------------------------------------------------------
+def oracle_sample_specs(wl, target_params):
+    """A sample of the workload with its tier mix: experts + backbone matrices + vectors + router."""
+    specs = wl.specs
+    ex = [k for k, s in enumerate(specs) if s.tier == 1]
+    bb2 = [k for k, s in enumerate(specs) if s.tier == 0 and len(s.shape) == 2 and s.numel <= 20_000_000]
+    vec = [k for k, s in enumerate(specs) if len(s.shape) == 1][:2]
+    rt = [k for k, s in enumerate(specs) if s.tier == 2]
+    chosen, tot = list(rt) + vec, sum(specs[k].numel for k in rt + vec)
+    bi = ei = 0
+    while tot < target_params and (bi < len(bb2) or ei < len(ex)):
+        # keep roughly the paper's 5 % backbone / 95 % expert split
+        nbb = sum(specs[k].numel for k in chosen if specs[k].tier == 0)
+        if bi < len(bb2) and nbb < 0.05 * tot:
+            k = bb2[bi]
+            bi += 1
+        elif ei < len(ex):
+            k = ex[ei]
+            ei += 1
+        else:
+            k = bb2[bi]
+            bi += 1
+        chosen.append(k)
+        tot += specs[k].numel
+    return chosen, tot
+
+
+def time_oracle(wl, tids, inputs, step, lr, seed):
+    import oracle as O
+    hpd = wl.hp
+    ohp = O.hparams(hpd.beta1, hpd.beta2, hpd.eps, hpd.clip_d, hpd.weight_decay)
+    states = {k: O.TensorState(wl.specs[k].shape, wl.specs[k].tier, hpd.policy, wl.specs[k].no_decay) for k in tids}
+    t0 = time.perf_counter()
+    for k in tids:
+        w, g = inputs[k]
+        O.tensor_step(w, g, states[k], k, ohp, step, lr, seed)
+    return time.perf_counter() - t0
+
+
+def cpu_inputs(wl, tids, step=1, src=None):
+    from paper_2607_19058_gb300 import workloads as WL
+    out = {}
+    for k in tids:
+        if src is not None:
+            w, g = src[k]
+            out[k] = (WL.bf16_bits(w).copy(), WL.bf16_bits(g).copy())
+        else:
+            out[k] = (WL.bf16_bits(WL.init_weight(wl, k, "cpu")).copy(), WL.bf16_bits(WL.grad(wl, k, step, "cpu")).copy())
+    return out
+
+
+def calibrate_oracle_rate(wl):
+    """Params/s of the oracle on a small expert-shaped tensor (to size the samples)."""
+    import numpy as np
+    import oracle as O
+    O.build()
+    n, m = 1024, 1024
+    rng = np.random.default_rng(0)
+    w = rng.integers(0, 2**16, n * m, dtype=np.uint16) & 0x3FFF
+    g = rng.integers(0, 2**16, n * m, dtype=np.uint16) & 0x3AFF
+    st = O.TensorState((n, m), O.TIER_EXPERT)
+    ohp = O.hparams(0.9, 0.999, 1e-30, 1.0, 0.1)
+    t0 = time.perf_counter()
+    O.tensor_step(w, g, st, 0, ohp, 1, 1e-3, 1)
+    return n * m / (time.perf_counter() - t0)
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    from paper_2607_19058_gb300 import workloads as WL
+    wl = WL.get(args.workload)
+    rate = calibrate_oracle_rate(wl)
+    per_step = max(1e6, rate * args.ref_seconds / max(1, args.steps + args.warmup))
+    tids, tot = oracle_sample_specs(wl, per_step)
+    inputs = cpu_inputs(wl, tids)
+    for s in range(args.warmup):
+        time_oracle(wl, tids, inputs, s + 1, wl.hp.lr, args.seed)
+    secs = [time_oracle(wl, tids, inputs, args.warmup + s + 1, wl.hp.lr, args.seed) for s in range(args.steps)]
+    value = tot * len(secs) / sum(secs)
+    ms_full = wl.numel / value * 1e3
+    desc = f"{len(tids)} of {len(wl.specs)} tensors ({tot} of {wl.numel} params, tier mix kept) per step"
+    out = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_full, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "params": wl.numel, "tensors": len(wl.specs), "policy": "tiered"},
+        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "note": "CPU oracle (plain fp64 C, single thread) on bounded samples of the workload; ms_per_step is the "
+                "full-workload equivalent at the sampled rate",
+    }
+    print(json.dumps(out))
+
+
+METRIC = "SkewAdam optimizer step over the 6.78B-parameter MoE shape set: params/s (step ms, HBM GB/s)"
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2607_19058_gb300 import _build
+    from paper_2607_19058_gb300 import skewadam as S
+    from paper_2607_19058_gb300 import workloads as WL
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    _build.build()
+    dev = torch.device("cuda", local)
+    wl = WL.get(args.workload)
+    hp = wl.hp
+    # inputs resident in HBM before timing
+    W = [WL.init_weight(wl, k, dev) for k in range(len(wl.specs))]
+    G = [WL.grad(wl, k, 1, dev) for k in range(len(wl.specs))]
+    params = [(W[k], G[k], s.tier, S.F_NO_DECAY if s.no_decay else 0) for k, s in enumerate(wl.specs)]
+    opt = S.SkewAdam(params, S.hparams(hp.beta1, hp.beta2, hp.eps, hp.clip_d, hp.weight_decay, hp.policy))
+    bm = byte_model(opt, len(wl.specs))
+    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+
+    step = 0
+    for _ in range(args.warmup):
+        step += 1
+        opt.step(step, hp.lr, args.seed)
+    opt.sync_status()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    clk = clocks_start(vis.split(",")[local] if vis else local)
+    S.skew_profile_begin(opt.h, args.steps)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step += 1
+        opt.step(step, hp.lr, args.seed)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = clocks_stop(clk)
+    opt.sync_status()
+    names, rows = S.skew_profile_end(opt.h)
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+
+    # per-kernel live durations
+    kmean = {n: statistics.fmean(r[i] for r in rows) for i, n in enumerate(names)}
+    dom = max(kmean, key=kmean.get)
+    peak, peak_src = peaks()
+    dom_bytes = bm["kernels"][dom]
+    achieved = dom_bytes / (kmean[dom] * 1e-3) / 1e9
+    step_gbs = bm["step_min"] / (ms * 1e-3) / 1e9
+
+    # end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e and args.e2e_steps > 0:
+        total = sum(w.numel() for w in W)
+        hg = torch.empty(total, dtype=torch.bfloat16, pin_memory=True)
+        hw = torch.empty(total, dtype=torch.bfloat16, pin_memory=True)
+        off = 0
+        views = []
+        for k in range(len(W)):
+            n = W[k].numel()
+            hg[off:off + n].copy_(G[k].reshape(-1))
+            views.append((hg[off:off + n].view(G[k].shape), hw[off:off + n].view(W[k].shape)))
+            off += n
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.e2e_steps):
+            step += 1
+            for k in range(len(W)):
+                G[k].copy_(views[k][0], non_blocking=True)
+            opt.step(step, hp.lr, args.seed)
+            for k in range(len(W)):
+                views[k][1].copy_(W[k], non_blocking=True)
+        b.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = a.elapsed_time(b) / args.e2e_steps
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": world * bm["N"] / (e2e_ms * 1e-3), "unit": "params/s", "ms_per_step": e2e_ms,
+               "h2d_bytes_per_step": 2 * bm["N"], "d2h_bytes_per_step": 2 * bm["N"],
+               "path": "skew_step via ctypes; gradients copied in from pinned host memory and weights read back "
+                       "to pinned host memory every step"}
+        del hg, hw, views
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        rate = calibrate_oracle_rate(wl)
+        tids, tot = oracle_sample_specs(wl, rate * args.cpu_seconds)
+        src = {k: (W[k], G[k]) for k in tids}
+        inputs = cpu_inputs(wl, tids, src=src)
+        secs = time_oracle(wl, tids, inputs, 1, hp.lr, args.seed)
+        cpu = {"value": tot / secs, "unit": "params/s", "cores": 1, "kind": "oracle",
+               "sample": f"one step of {len(tids)} of the {len(wl.specs)} tensors ({tot} params, tier mix kept) "
+                         f"in {secs:.1f} s, single-threaded fp64 C"}
+
+    if rank == 0:
+        out = {
+            "metric": METRIC,
+            "value": world * bm["N"] / (ms * 1e-3), "unit": "params/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": wl.name, "params": bm["N"], "tensors": len(wl.specs), "policy": "tiered",
+                       "state_bytes": opt.state_bytes, "workspace_bytes": opt.workspace_bytes,
+                       "l2": "inputs larger than L2 (27.1 GB of bf16 weights + grads vs 129 MiB), no flush",
+                       "weights_grads": "bf16, W~N(0,0.02^2), G~N(0,1e-3^2)"},
+            "hbm": {"min_bytes_per_step": bm["step_min"], "achieved_gbs": step_gbs,
+                    "frac_of_8tbs": step_gbs / NOMINAL_HBM_GBS, "frac_of_measured": step_gbs / peak,
+                    "peak_gbs": peak, "peak_source": peak_src},
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None, "algorithmic_bytes_per_launch": dom_bytes,
+                         "launch_ms": kmean[dom], "peak_source": peak_src},
+            "kernels_ms": kmean,
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+            "gpu_launches": args.steps * len(names),
+            "clocks": clocks,
+        }
+        print(json.dumps(out))
+    opt.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,232 @@
+/*
+ * libskewadam -- the SkewAdam optimizer step (tiered optimizer state for MoE
+ * training) on one NVIDIA GB300 (sm_103a).
+ *
+ * The step follows "Where Should Optimizer State Live? Tiered State Allocation
+ * for Memory-Efficient MoE Training":
+ *   - tiers (Sec. 3 "The tiers", Fig. 1): backbone tensors keep fp32 momentum
+ *     and a factored second moment; expert tensors keep only the factored
+ *     second moment; the router keeps the exact (unfactored) second moment and
+ *     no weight decay; any vector (1-D tensor) keeps the exact second moment
+ *     (Algorithm 1);
+ *   - factored second moment (Eq. 1): per matrix W (n x m) an fp32 row vector
+ *     R (n) and column vector C (m) of exponential moving averages of the row
+ *     and column means of G*G; Vhat = R C^T / mean(R);
+ *   - update (Algorithm 1): D = sqrt(max(Vhat, eps)); backbone
+ *     U = sqrt(1-beta2^t)/(1-beta1^t) * M / D with M = beta1 M + (1-beta1) G;
+ *     other tiers U = sqrt(1-beta2^t) * G / D;
+ *   - update clipping (Sec. 3 "Update clipping and low-precision updates"):
+ *     U <- U / max(1, RMS(U)/d), RMS over the whole tensor;
+ *   - decoupled weight decay fused into the fp32 update ahead of the cast
+ *     (Sec. 3 footnote, Sec. 5): x = w (1 - lr*lambda) - lr * U;
+ *   - dithered bf16 write-back (Sec. 3, Algorithm 1 last line): the fp32 value
+ *     x is rounded to bf16 by adding a uniform 16-bit integer r to its bit
+ *     pattern and truncating (unbiased stochastic rounding with the exact bf16
+ *     ulp of x); r is a Philox-4x32-10 draw keyed by (seed) and counted by
+ *     (element index / 8, tensor id, step), so a step is bit-reproducible;
+ *   - state size (Sec. 3 "Memory model", Eq. 2, App. B Table 5): 4 bytes per
+ *     momentum element, per exact-second-moment element and per R / C entry.
+ *
+ * Conventions for every entry point:
+ *   - Return SKEW_OK (0) or a negative SKEW_E* code; nothing aborts or throws.
+ *     skew_last_error() gives a one-line reason for the last failure on a
+ *     handle (skew_create failures: pass NULL).
+ *   - Device memory (weights, gradients, state, workspace) is owned by the
+ *     caller; the library owns only host-side metadata in the handle.
+ *   - Pointers passed as `void *stream` are cudaStream_t values (0 = legacy
+ *     default stream). Work is enqueued asynchronously on that stream; one
+ *     stream per handle at a time.
+ *   - Element counts are 64-bit; a tensor may exceed 2^31 elements.
+ */
+#ifndef SKEWADAM_H_
+#define SKEWADAM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes -------------------------------------------------------- */
+#define SKEW_OK 0
+#define SKEW_EINVAL (-1)   /* invalid argument (null, shape, tier, hyper-parameter, step, size) */
+#define SKEW_ENOMEM (-2)   /* host allocation failed                                        */
+#define SKEW_ECUDA (-3)    /* a CUDA runtime call failed                                   */
+#define SKEW_ETIMEOUT (-4) /* a bounded device-side wait gave up (see skew_sync_status)    */
+#define SKEW_ESTATE (-5)   /* call out of order (e.g. skew_step before skew_bind)          */
+
+/* ---- tiers (Sec. 3 "The tiers") -------------------------------------------- */
+#define SKEW_TIER_BACKBONE 0 /* embeddings, positions, attention, dense FFN, norms */
+#define SKEW_TIER_EXPERT 1   /* expert matrices                                     */
+#define SKEW_TIER_ROUTER 2   /* the gate                                            */
+
+/* ---- allocation policies: the paper's policy and the Table 3 variants ------ */
+#define SKEW_POLICY_TIERED 0          /* SkewAdam as published                         */
+#define SKEW_POLICY_EXPERT_MOMENTUM 1 /* "+ momentum on experts"                        */
+#define SKEW_POLICY_FACTORED_ROUTER 2 /* "factored router"                              */
+#define SKEW_POLICY_UNIFORM 3         /* "uniform (momentum + factored)" on every tier  */
+
+/* ---- per-tensor flags ------------------------------------------------------ */
+#define SKEW_F_NO_DECAY 1u /* exempt this tensor from weight decay (the router always is) */
+
+/* ---- second-moment kinds reported by skew_tensor_info ----------------------- */
+#define SKEW_KIND_FULL 0     /* exact second moment v (router, vectors)  */
+#define SKEW_KIND_FACTORED 1 /* row / column factors R, C (Eq. 1)        */
+
+typedef struct skew_handle skew_handle_t; /* opaque */
+
+/*
+ * One parameter tensor. The tensor id used by the dither is its index in the
+ * array passed to skew_create.
+ *   weight : device pointer to the bf16 weights, contiguous row-major, updated
+ *            in place by skew_step; 2-byte aligned (16-byte alignment enables
+ *            the vectorised path). Borrowed: must stay valid while the handle
+ *            is bound.
+ *   grad   : device pointer to the bf16 gradient, same shape and layout; read
+ *            only. Borrowed like `weight`.
+ *   shape  : shape[0] = rows n (>= 1); shape[1] = columns m (>= 1) when
+ *            ndim == 2, ignored when ndim == 1.
+ *   ndim   : 1 (vector) or 2 (matrix).
+ *   tier   : SKEW_TIER_*.
+ *   flags  : SKEW_F_* bits.
+ *   reserved: must be 0.
+ */
+typedef struct {
+    void *weight;
+    const void *grad;
+    int64_t shape[2];
+    int32_t ndim;
+    int32_t tier;
+    uint32_t flags;
+    uint32_t reserved;
+} skew_param_desc_t;
+
+/*
+ * Hyper-parameters (Algorithm 1, App. A Table 9). The paper's defaults are
+ * beta1 = 0.9, beta2 = 0.999, eps = 1e-8, clip_d = 1, weight_decay = 0.05.
+ *   0 <= beta1 < 1, 0 <= beta2 < 1, eps > 0 (finite), clip_d > 0 (finite),
+ *   weight_decay >= 0 (finite), policy = SKEW_POLICY_*.
+ */
+typedef struct {
+    float beta1;
+    float beta2;
+    float eps;
+    float clip_d;
+    float weight_decay;
+    int32_t policy;
+} skew_hparams_t;
+
+/*
+ * Where one tensor's state lives inside the caller's state buffer (offsets in
+ * fp32 elements from its start; -1 when the tensor has no such array).
+ *   m_offset: momentum M (numel floats, row-major)
+ *   v_offset: exact second moment v (numel floats)
+ *   r_offset: R (rows floats), c_offset: C (cols floats)
+ */
+typedef struct {
+    int32_t kind;       /* SKEW_KIND_*                                         */
+    int32_t momentum;   /* 1 if the tensor keeps fp32 momentum                 */
+    int32_t decay;      /* 1 if weight decay applies                           */
+    int32_t vectorized; /* 1 if the 16-byte vector path serves it (after bind) */
+    int64_t rows, cols, numel;
+    int64_t m_offset, v_offset, r_offset, c_offset;
+} skew_tensor_info_t;
+
+/*
+ * Plans the step for `n_params` tensors (n_params >= 0; 0 gives a handle whose
+ * step does nothing). Validates every descriptor and the hyper-parameters,
+ * resolves each tensor's tier policy (kind / momentum / decay), lays out the
+ * optimizer state and the workspace. Host only: no CUDA call, no device
+ * memory touched. On success *out receives a new handle (free with
+ * skew_destroy). Errors: SKEW_EINVAL (reason in skew_last_error(NULL)),
+ * SKEW_ENOMEM.
+ */
+int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hparams_t *hp,
+                skew_handle_t **out);
+
+/* Frees the handle's host metadata (not the caller's device memory). NULL is a no-op. */
+int skew_destroy(skew_handle_t *h);
+
+/*
+ * Exact optimizer-state size in bytes: 4 * (sum over momentum tensors of numel
+ * + sum over factored tensors of (rows + cols) + sum over exact-second-moment
+ * tensors of numel) -- Eq. 2 with the vectors' full v of Table 5. The caller
+ * allocates exactly this many bytes of device memory for the state. 0 for NULL.
+ */
+size_t skew_state_bytes(const skew_handle_t *h);
+
+/*
+ * Scratch the step needs besides the state (per-tensor partial sums, scalars,
+ * descriptor and tile tables). Not optimizer state. 0 for NULL.
+ */
+size_t skew_workspace_bytes(const skew_handle_t *h);
+
+/*
+ * Binds caller-owned device buffers to the handle: `state` (exactly
+ * skew_state_bytes bytes) and `workspace` (exactly skew_workspace_bytes bytes),
+ * both 256-byte aligned device pointers (NULL allowed when the size is 0).
+ * Uploads the descriptor and tile tables into the workspace and zero-fills the
+ * state (the paper's initial M = v = R = C = 0), enqueued on `stream`.
+ * May be called again to re-bind (the state is zeroed again).
+ * Errors: SKEW_EINVAL (size / alignment), SKEW_ECUDA.
+ */
+int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace, size_t workspace_bytes,
+              void *stream);
+
+/*
+ * Enqueues one SkewAdam step over every tensor on `stream`: reads each
+ * gradient, updates the state and writes the bf16 weights in place.
+ *   step : global 1-based step t (bias corrections beta^t; the dither counter
+ *          uses its low 32 bits). All tensors advance together.
+ *   lr   : the scheduled learning rate eta_t (finite, >= 0); the caller owns
+ *          the schedule.
+ *   seed : 64-bit dither seed.
+ * Asynchronous: device-side problems are reported by skew_sync_status.
+ * Errors: SKEW_ESTATE (not bound), SKEW_EINVAL (step < 1, lr not finite or
+ * negative), SKEW_ECUDA (launch failure).
+ */
+int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *stream);
+
+/*
+ * Synchronises `stream` and reports the device-side status word of the last
+ * steps: SKEW_OK, or SKEW_ETIMEOUT if a bounded device wait gave up (the word
+ * is cleared by this call). Errors: SKEW_ESTATE, SKEW_ECUDA.
+ */
+int skew_sync_status(skew_handle_t *h, void *stream);
+
+/*
+ * Per-tensor scalars of the last completed step, for inspection and tests:
+ * out[0] = mean(R) (factored tensors, else 0), out[1] = sum of U^2 over the
+ * tensor, out[2] = RMS(U), out[3] = clip factor 1/max(1, RMS/d). Synchronises
+ * `stream`. Errors: SKEW_EINVAL (tid), SKEW_ESTATE, SKEW_ECUDA.
+ */
+int skew_tensor_scalars(skew_handle_t *h, int32_t tid, double out[4], void *stream);
+
+/* Resolved policy and state offsets of tensor `tid`. Errors: SKEW_EINVAL. */
+int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *out);
+
+/*
+ * Benchmark support: per-kernel timing. After skew_profile_begin(h, n), each of
+ * the next n calls of skew_step records a CUDA event before and after every
+ * kernel it launches (on the step's stream; no extra synchronisation).
+ * skew_profile_end(h, ms, cap, &steps, &kernels) synchronises, writes the
+ * durations in milliseconds row-major into ms[steps][kernels] (up to cap
+ * values), releases the events and stops recording. skew_kernel_name(k) names
+ * kernel k of a step. Errors: SKEW_EINVAL, SKEW_ECUDA.
+ */
+int skew_profile_begin(skew_handle_t *h, int32_t max_steps);
+int skew_profile_end(skew_handle_t *h, double *ms, int64_t cap, int32_t *n_steps, int32_t *n_kernels);
+const char *skew_kernel_name(int32_t k);
+
+/* Number of tensors the handle plans for (0 for NULL). */
+int32_t skew_num_tensors(const skew_handle_t *h);
+
+/* One-line reason for the last failure on `h` (or of skew_create when h is NULL). */
+const char *skew_last_error(const skew_handle_t *h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SKEWADAM_H_ */

@@ -1,0 +1,471 @@
+// Host side of libskewadam: validation, tier policy, state / workspace layout,
+// descriptor and tile tables, and the C ABI declared in include/skewadam.h.
+//
+// The tier policy follows Sec. 3 "The tiers" and Algorithm 1 (vectors keep the
+// exact second moment; the router keeps it and no weight decay; backbone keeps
+// fp32 momentum), with the Table 3 variants selected by skew_hparams_t.policy.
+// The state layout realises Eq. 2 (plus the vectors' full v, Table 5) with no
+// padding, so skew_state_bytes() is the closed form exactly.
+#include "skewadam.h"
+#include "skew_plan.h"
+
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+using namespace skew;
+
+namespace {
+
+struct TPlan {
+    int kind = 0, momentum = 0, decay = 0, vec = 0;
+    int64_t n = 0, m = 0, numel = 0;
+    int64_t moff = -1, voff = -1, roff = -1, coff = -1;  // floats into the state
+    uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
+    size_t ws_rowp = 0, ws_colp = 0, ws_bsc = 0, ws_rsum = 0, ws_u2 = 0;  // bytes into the workspace
+};
+
+thread_local std::string g_create_err;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace
+
+struct skew_handle {
+    std::vector<skew_param_desc_t> desc;
+    skew_hparams_t hp{};
+    std::vector<TPlan> t;
+    size_t state_bytes = 0, ws_bytes = 0;
+    size_t ws_scal = 0, ws_err = 0, ws_tab = 0, ws_tab_end = 0;
+    size_t ws_tens = 0, ws_itemsA = 0, ws_itemsF = 0, ws_itemsBC = 0;
+    std::vector<uint2> itemsA, itemsF, itemsBC;
+    char *state = nullptr, *ws = nullptr;
+    bool bound = false;
+    std::string err;
+    // per-kernel timing (skew_profile_begin / skew_profile_end)
+    std::vector<cudaEvent_t> prof_ev;
+    int32_t prof_max = 0, prof_used = 0;
+    ~skew_handle() {
+        for (cudaEvent_t e : prof_ev) cudaEventDestroy(e);
+    }
+};
+
+static int fail(skew_handle_t *h, int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (h)
+        h->err = buf;
+    else
+        g_create_err = buf;
+    return code;
+}
+
+static int cuda_fail(skew_handle_t *h, cudaError_t e, const char *what) {
+    return fail(h, SKEW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Tier policy: (kind, momentum, decay) of one tensor.
+static void resolve(int ndim, int tier, int policy, uint32_t flags, TPlan &p) {
+    if (ndim == 1)
+        p.kind = kKindFull;  // Algorithm 1: a vector keeps the full second moment
+    else if (tier == SKEW_TIER_ROUTER && policy != SKEW_POLICY_FACTORED_ROUTER && policy != SKEW_POLICY_UNIFORM)
+        p.kind = kKindFull;  // the router keeps the exact second moment
+    else
+        p.kind = kKindFactored;  // Eq. 1
+    if (tier == SKEW_TIER_BACKBONE)
+        p.momentum = 1;
+    else if (tier == SKEW_TIER_EXPERT)
+        p.momentum = (policy == SKEW_POLICY_EXPERT_MOMENTUM || policy == SKEW_POLICY_UNIFORM);
+    else
+        p.momentum = (policy == SKEW_POLICY_UNIFORM);
+    p.decay = (tier != SKEW_TIER_ROUTER) && !(flags & SKEW_F_NO_DECAY);
+}
+
+// Tile geometry: a factored tile is (tile_rows rows) x (8*LC columns), a full
+// tile is 32 Ki flat elements.
+static void geometry(TPlan &p) {
+    if (p.kind == kKindFactored) {
+        int64_t vecs = (p.m + 7) / 8;  // 8-column groups per row
+        uint32_t lc = 1, lcl = 0;
+        while (lc < 32 && lc < vecs) {
+            lc <<= 1;
+            ++lcl;
+        }
+        p.lcl = lcl;
+        p.strips = (uint32_t)((p.m + 8 * lc - 1) / (8 * lc));
+        p.tile_rows = (uint32_t)(kVecPerThread * (kThreads / lc));
+        p.rowtiles = (uint32_t)((p.n + p.tile_rows - 1) / p.tile_rows);
+        p.ntiles = p.strips * p.rowtiles;
+        p.nfr = (uint32_t)((p.n + kFinChunk - 1) / kFinChunk);
+        p.nfc = (uint32_t)((p.m + kFinChunk - 1) / kFinChunk);
+    } else {
+        p.lcl = 0;
+        p.strips = 1;
+        p.tile_rows = 0;
+        p.rowtiles = (uint32_t)((p.numel + kFlatTileElems - 1) / kFlatTileElems);
+        p.ntiles = p.rowtiles;
+        p.nfr = p.nfc = 0;
+    }
+}
+
+extern "C" {
+
+int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hparams_t *hp, skew_handle_t **out) {
+    g_create_err.clear();
+    if (!out) return fail(nullptr, SKEW_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (!hp) return fail(nullptr, SKEW_EINVAL, "hp is NULL");
+    if (n_params < 0 || (n_params > 0 && !params)) return fail(nullptr, SKEW_EINVAL, "bad parameter list");
+    const skew_hparams_t H = *hp;
+    auto finite = [](float x) { return std::isfinite(x); };
+    if (!finite(H.beta1) || H.beta1 < 0.f || H.beta1 >= 1.f) return fail(nullptr, SKEW_EINVAL, "beta1 must be in [0,1)");
+    if (!finite(H.beta2) || H.beta2 < 0.f || H.beta2 >= 1.f) return fail(nullptr, SKEW_EINVAL, "beta2 must be in [0,1)");
+    if (!finite(H.eps) || !(H.eps > 0.f)) return fail(nullptr, SKEW_EINVAL, "eps must be finite and > 0");
+    if (!finite(H.clip_d) || !(H.clip_d > 0.f)) return fail(nullptr, SKEW_EINVAL, "clip_d must be finite and > 0");
+    if (!finite(H.weight_decay) || H.weight_decay < 0.f) return fail(nullptr, SKEW_EINVAL, "weight_decay must be finite and >= 0");
+    if (H.policy < SKEW_POLICY_TIERED || H.policy > SKEW_POLICY_UNIFORM) return fail(nullptr, SKEW_EINVAL, "unknown policy %d", H.policy);
+
+    skew_handle *h = new (std::nothrow) skew_handle();
+    if (!h) return fail(nullptr, SKEW_ENOMEM, "out of host memory");
+    try {
+        h->hp = H;
+        h->desc.assign(params, params + n_params);
+        h->t.resize(n_params);
+    } catch (...) {
+        delete h;
+        return fail(nullptr, SKEW_ENOMEM, "out of host memory");
+    }
+    const int64_t kMaxExtent = int64_t(1) << 40;
+    for (int32_t k = 0; k < n_params; ++k) {
+        const skew_param_desc_t &d = params[k];
+        TPlan &p = h->t[k];
+        if (!d.weight || !d.grad) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: null weight or grad", k); }
+        if (((uintptr_t)d.weight & 1) || ((uintptr_t)d.grad & 1)) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: bf16 pointers must be 2-byte aligned", k); }
+        if (d.ndim != 1 && d.ndim != 2) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: ndim must be 1 or 2", k); }
+        if (d.tier < SKEW_TIER_BACKBONE || d.tier > SKEW_TIER_ROUTER) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: unknown tier %d", k, d.tier); }
+        if (d.flags & ~SKEW_F_NO_DECAY) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: unknown flags", k); }
+        if (d.reserved != 0) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: reserved must be 0", k); }
+        p.n = d.shape[0];
+        p.m = d.ndim == 2 ? d.shape[1] : 1;
+        if (p.n < 1 || p.m < 1 || p.n > kMaxExtent || p.m > kMaxExtent) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: extents must be in [1, 2^40]", k); }
+        if (p.n > (int64_t(1) << 62) / p.m) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: too many elements", k); }
+        p.numel = p.n * p.m;
+        resolve(d.ndim, d.tier, H.policy, d.flags, p);
+        geometry(p);
+    }
+
+    // State layout (fp32 offsets): [momentum arrays][full v arrays][R arrays][C arrays].
+    // Arrays whose length is a multiple of 4 come first in each group so that as
+    // many as possible start on a 16-byte boundary; there is no padding.
+    int64_t off = 0;
+    for (int pass = 0; pass < 2; ++pass)
+        for (auto &p : h->t)
+            if (p.momentum && ((p.numel % 4 == 0) == (pass == 0))) { p.moff = off; off += p.numel; }
+    for (int pass = 0; pass < 2; ++pass)
+        for (auto &p : h->t)
+            if (p.kind == kKindFull && ((p.numel % 4 == 0) == (pass == 0))) { p.voff = off; off += p.numel; }
+    for (auto &p : h->t)
+        if (p.kind == kKindFactored) { p.roff = off; off += p.n; }
+    for (auto &p : h->t)
+        if (p.kind == kKindFactored) { p.coff = off; off += p.m; }
+    h->state_bytes = size_t(off) * 4;
+
+    // Work items of the three phases.
+    try {
+        for (int32_t k = 0; k < n_params; ++k) {
+            const TPlan &p = h->t[k];
+            if (p.kind == kKindFactored) {
+                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(k, i));
+                for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(k, i));
+            }
+            for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsBC.push_back(make_uint2(k, i));
+        }
+    } catch (...) {
+        delete h;
+        return fail(nullptr, SKEW_ENOMEM, "out of host memory");
+    }
+
+    // Workspace layout (bytes, 256-aligned regions).
+    size_t w = 0;
+    h->ws_scal = w;
+    w = align_up(w + sizeof(TensorScal) * n_params, 256);
+    h->ws_err = w;
+    w = align_up(w + 16, 256);
+    h->ws_tab = w;
+    h->ws_tens = w;
+    w = align_up(w + sizeof(TensorDev) * n_params, 256);
+    h->ws_itemsA = w;
+    w = align_up(w + sizeof(uint2) * h->itemsA.size(), 256);
+    h->ws_itemsF = w;
+    w = align_up(w + sizeof(uint2) * h->itemsF.size(), 256);
+    h->ws_itemsBC = w;
+    w = align_up(w + sizeof(uint2) * h->itemsBC.size(), 256);
+    h->ws_tab_end = w;
+    for (auto &p : h->t) {
+        if (p.kind == kKindFactored) {
+            p.ws_rowp = w; w = align_up(w + 4 * size_t(p.strips) * p.n, 256);
+            p.ws_colp = w; w = align_up(w + 4 * size_t(p.rowtiles) * p.m, 256);
+            p.ws_bsc = w;  w = align_up(w + 4 * size_t(p.m), 256);
+            p.ws_rsum = w; w = align_up(w + 8 * size_t(p.nfr), 256);
+        }
+        p.ws_u2 = w;
+        w = align_up(w + 4 * size_t(p.ntiles), 256);
+    }
+    h->ws_bytes = w;
+    *out = h;
+    return SKEW_OK;
+}
+
+int skew_destroy(skew_handle_t *h) {
+    delete h;
+    return SKEW_OK;
+}
+
+size_t skew_state_bytes(const skew_handle_t *h) { return h ? h->state_bytes : 0; }
+
+size_t skew_workspace_bytes(const skew_handle_t *h) { return h ? h->ws_bytes : 0; }
+
+int32_t skew_num_tensors(const skew_handle_t *h) { return h ? (int32_t)h->t.size() : 0; }
+
+const char *skew_last_error(const skew_handle_t *h) { return h ? h->err.c_str() : g_create_err.c_str(); }
+
+int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *out) {
+    if (!h || !out) return SKEW_EINVAL;
+    if (tid < 0 || tid >= (int32_t)h->t.size()) return fail(const_cast<skew_handle_t *>(h), SKEW_EINVAL, "tid %d out of range", tid);
+    const TPlan &p = h->t[tid];
+    out->kind = p.kind;
+    out->momentum = p.momentum;
+    out->decay = p.decay;
+    out->vectorized = p.vec;
+    out->rows = p.n;
+    out->cols = p.m;
+    out->numel = p.numel;
+    out->m_offset = p.moff;
+    out->v_offset = p.voff;
+    out->r_offset = p.roff;
+    out->c_offset = p.coff;
+    return SKEW_OK;
+}
+
+int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace, size_t workspace_bytes, void *stream) {
+    if (!h) return SKEW_EINVAL;
+    if (state_bytes != h->state_bytes) return fail(h, SKEW_EINVAL, "state buffer is %zu bytes, need exactly %zu", state_bytes, h->state_bytes);
+    if (workspace_bytes != h->ws_bytes) return fail(h, SKEW_EINVAL, "workspace is %zu bytes, need exactly %zu", workspace_bytes, h->ws_bytes);
+    if ((h->state_bytes && !state) || (h->ws_bytes && !workspace)) return fail(h, SKEW_EINVAL, "null device buffer");
+    if (((uintptr_t)state & 255) || ((uintptr_t)workspace & 255)) return fail(h, SKEW_EINVAL, "state and workspace must be 256-byte aligned");
+    cudaStream_t s = (cudaStream_t)stream;
+    h->state = (char *)state;
+    h->ws = (char *)workspace;
+    h->bound = false;
+
+    // Host image of [TensorDev table][item tables].
+    std::vector<char> img;
+    try {
+        img.assign(h->ws_tab_end - h->ws_tab, 0);
+    } catch (...) {
+        return fail(h, SKEW_ENOMEM, "out of host memory");
+    }
+    TensorDev *td = reinterpret_cast<TensorDev *>(img.data() + (h->ws_tens - h->ws_tab));
+    float *sf = reinterpret_cast<float *>(state);
+    auto al16 = [](const void *p) { return ((uintptr_t)p & 15) == 0; };
+    for (size_t k = 0; k < h->t.size(); ++k) {
+        TPlan &p = h->t[k];
+        const skew_param_desc_t &d = h->desc[k];
+        TensorDev &T = td[k];
+        T.w = (uint16_t *)d.weight;
+        T.g = (const uint16_t *)d.grad;
+        T.M = p.moff >= 0 ? sf + p.moff : nullptr;
+        T.v = p.voff >= 0 ? sf + p.voff : nullptr;
+        T.R = p.roff >= 0 ? sf + p.roff : nullptr;
+        T.C = p.coff >= 0 ? sf + p.coff : nullptr;
+        T.rowp = p.kind == kKindFactored ? (float *)(h->ws + p.ws_rowp) : nullptr;
+        T.colp = p.kind == kKindFactored ? (float *)(h->ws + p.ws_colp) : nullptr;
+        T.bsc = p.kind == kKindFactored ? (float *)(h->ws + p.ws_bsc) : nullptr;
+        T.rsum = p.kind == kKindFactored ? (double *)(h->ws + p.ws_rsum) : nullptr;
+        T.u2 = (float *)(h->ws + p.ws_u2);
+        T.n = p.n;
+        T.m = p.m;
+        T.numel = p.numel;
+        T.tid = (uint32_t)k;
+        T.kind = p.kind;
+        T.momentum = p.momentum;
+        T.decay = p.decay;
+        bool vec = al16(T.w) && al16(T.g) && (!T.M || al16(T.M));
+        if (p.kind == kKindFull)
+            vec = vec && (p.numel % 8 == 0) && al16(T.v);
+        else
+            vec = vec && (p.m % 8 == 0);
+        p.vec = vec ? 1 : 0;
+        T.vec = p.vec;
+        T.lcl = p.lcl;
+        T.strips = p.strips;
+        T.rowtiles = p.rowtiles;
+        T.tile_rows = p.tile_rows;
+        T.ntiles = p.ntiles;
+        T.nfr = p.nfr;
+        T.nfc = p.nfc;
+    }
+    auto put = [&](size_t at, const std::vector<uint2> &v) {
+        if (!v.empty()) std::memcpy(img.data() + (at - h->ws_tab), v.data(), v.size() * sizeof(uint2));
+    };
+    put(h->ws_itemsA, h->itemsA);
+    put(h->ws_itemsF, h->itemsF);
+    put(h->ws_itemsBC, h->itemsBC);
+
+    cudaError_t e;
+    if (!img.empty()) {
+        e = cudaMemcpyAsync(h->ws + h->ws_tab, img.data(), img.size(), cudaMemcpyHostToDevice, s);
+        if (e != cudaSuccess) return cuda_fail(h, e, "upload of descriptor tables");
+        // the pageable source may be freed on return only once the copy has been staged
+        e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess) return cuda_fail(h, e, "upload of descriptor tables");
+    }
+    if (h->state_bytes) {
+        e = cudaMemsetAsync(state, 0, h->state_bytes, s);
+        if (e != cudaSuccess) return cuda_fail(h, e, "zero-fill of the state");
+    }
+    if (h->ws_bytes) {
+        e = cudaMemsetAsync(h->ws + h->ws_scal, 0, h->ws_tab - h->ws_scal, s);
+        if (e != cudaSuccess) return cuda_fail(h, e, "zero-fill of the scalars");
+    }
+    h->bound = true;
+    return SKEW_OK;
+}
+
+int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *stream) {
+    if (!h) return SKEW_EINVAL;
+    if (!h->bound) return fail(h, SKEW_ESTATE, "skew_step before skew_bind");
+    if (step < 1) return fail(h, SKEW_EINVAL, "step must be >= 1 (got %lld)", (long long)step);
+    if (!std::isfinite(lr) || lr < 0.f) return fail(h, SKEW_EINVAL, "lr must be finite and >= 0");
+    if (h->t.empty()) return SKEW_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    const skew_hparams_t &H = h->hp;
+    const double t = (double)step;
+    const double bc1 = 1.0 - std::pow((double)H.beta1, t);
+    const double s2 = std::sqrt(1.0 - std::pow((double)H.beta2, t));
+
+    StepArgs a{};
+    a.tensors = reinterpret_cast<const TensorDev *>(h->ws + h->ws_tens);
+    a.scal = reinterpret_cast<TensorScal *>(h->ws + h->ws_scal);
+    a.err = reinterpret_cast<uint32_t *>(h->ws + h->ws_err);
+    a.b1 = H.beta1;
+    a.b2 = H.beta2;
+    a.c1 = (float)(1.0 - (double)H.beta1);
+    a.c2 = (float)(1.0 - (double)H.beta2);
+    a.ce = (float)(1.0 / std::sqrt((double)H.eps));
+    a.wdf = (float)(1.0 - (double)lr * (double)H.weight_decay);
+    a.lr = lr;
+    a.clip_d = H.clip_d;
+    a.coef_mom = s2 / bc1;
+    a.coef_plain = s2;
+    a.step_lo = (uint32_t)(uint64_t)step;
+    a.seed_lo = (uint32_t)seed;
+    a.seed_hi = (uint32_t)(seed >> 32);
+
+    LaunchPlan lp{};
+    lp.nA = (uint32_t)h->itemsA.size();
+    lp.nF = (uint32_t)h->itemsF.size();
+    lp.nBC = (uint32_t)h->itemsBC.size();
+    lp.itemsA = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsA);
+    lp.itemsF = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsF);
+    lp.itemsBC = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsBC);
+
+    if (h->prof_used < h->prof_max) {
+        lp.events = reinterpret_cast<void *const *>(h->prof_ev.data() + size_t(h->prof_used) * (kNumKernels + 1));
+        ++h->prof_used;
+    }
+    cudaError_t e = cudaMemsetAsync(h->ws + h->ws_scal, 0, sizeof(TensorScal) * h->t.size(), s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "reset of per-step scalars");
+    e = (cudaError_t)launch_step(lp, a, stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
+    return SKEW_OK;
+}
+
+int skew_profile_begin(skew_handle_t *h, int32_t max_steps) {
+    if (!h || max_steps < 0 || max_steps > (1 << 20)) return SKEW_EINVAL;
+    for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
+    h->prof_ev.clear();
+    h->prof_max = h->prof_used = 0;
+    try {
+        h->prof_ev.resize(size_t(max_steps) * (kNumKernels + 1), nullptr);
+    } catch (...) {
+        return fail(h, SKEW_ENOMEM, "out of host memory");
+    }
+    for (auto &ev : h->prof_ev) {
+        cudaError_t e = cudaEventCreate(&ev);
+        if (e != cudaSuccess) {
+            ev = nullptr;
+            return cuda_fail(h, e, "event create");
+        }
+    }
+    h->prof_max = max_steps;
+    return SKEW_OK;
+}
+
+int skew_profile_end(skew_handle_t *h, double *ms, int64_t cap, int32_t *n_steps, int32_t *n_kernels) {
+    if (!h || (cap > 0 && !ms)) return SKEW_EINVAL;
+    int rc = SKEW_OK;
+    int64_t w = 0;
+    for (int32_t st = 0; st < h->prof_used; ++st) {
+        cudaEvent_t *ev = h->prof_ev.data() + size_t(st) * (kNumKernels + 1);
+        for (int k = 0; k < kNumKernels; ++k) {
+            float t = 0.f;
+            cudaError_t e = cudaEventSynchronize(ev[k + 1]);
+            if (e == cudaSuccess) e = cudaEventElapsedTime(&t, ev[k], ev[k + 1]);
+            if (e != cudaSuccess && rc == SKEW_OK) rc = cuda_fail(h, e, "event timing");
+            if (w < cap) ms[w] = t;
+            ++w;
+        }
+    }
+    if (n_steps) *n_steps = h->prof_used;
+    if (n_kernels) *n_kernels = kNumKernels;
+    for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
+    h->prof_ev.clear();
+    h->prof_max = h->prof_used = 0;
+    return rc;
+}
+
+const char *skew_kernel_name(int32_t k) { return (k >= 0 && k < kNumKernels) ? kKernelNames[k] : ""; }
+
+int skew_sync_status(skew_handle_t *h, void *stream) {
+    if (!h) return SKEW_EINVAL;
+    if (!h->bound) return fail(h, SKEW_ESTATE, "not bound");
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "stream synchronize");
+    uint32_t word = 0;
+    e = cudaMemcpy(&word, h->ws + h->ws_err, 4, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(h, e, "status read");
+    if (word) {
+        cudaMemset(h->ws + h->ws_err, 0, 4);
+        return fail(h, SKEW_ETIMEOUT, "device wait gave up (status 0x%x)", word);
+    }
+    return SKEW_OK;
+}
+
+int skew_tensor_scalars(skew_handle_t *h, int32_t tid, double out[4], void *stream) {
+    if (!h || !out) return SKEW_EINVAL;
+    if (tid < 0 || tid >= (int32_t)h->t.size()) return fail(h, SKEW_EINVAL, "tid %d out of range", tid);
+    if (!h->bound) return fail(h, SKEW_ESTATE, "not bound");
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "stream synchronize");
+    TensorScal sc;
+    e = cudaMemcpy(&sc, h->ws + h->ws_scal + sizeof(TensorScal) * tid, sizeof sc, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(h, e, "scalar read");
+    out[0] = sc.rbar;
+    out[1] = sc.sumsq;
+    out[2] = sc.rms;
+    out[3] = sc.kappa;
+    return SKEW_OK;
+}
+
+}  // extern "C"

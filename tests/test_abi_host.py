@@ -1,0 +1,177 @@
+"""Host-side checks of the C ABI (no GPU needed: no compute call is made).
+
+The library must load, export every function include/skewadam.h declares, and
+its ctypes structs must have the header's layout. skew_create is host-only
+planning, so tiering, the closed-form state size, the state layout and the
+argument validation are all checked here on the CPU.
+"""
+import ctypes as C
+import os
+import re
+import subprocess
+import tempfile
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2607_19058_gb300 import _build
+from paper_2607_19058_gb300 import skewadam as S
+from paper_2607_19058_gb300 import workloads as WL
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "skewadam.h")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    _build.build()
+    return S.load()
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(skew_[a-z_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _declared()
+    assert set(names) == set(S.EXPORTS)
+    out = subprocess.run(["nm", "-D", "--defined-only", S.LIB_PATH], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (skew_\w+)", out))
+    for n in names:
+        assert n in exported, n
+        assert hasattr(lib, n)
+
+
+def test_struct_layout_matches_header():
+    prog = r'''
+    #include <stdio.h>
+    #include <stddef.h>
+    #include "skewadam.h"
+    int main(void) {
+      printf("%zu %zu %zu %zu %zu %zu %zu\n", sizeof(skew_param_desc_t), sizeof(skew_hparams_t),
+             sizeof(skew_tensor_info_t), offsetof(skew_param_desc_t, shape), offsetof(skew_param_desc_t, ndim),
+             offsetof(skew_param_desc_t, flags), offsetof(skew_tensor_info_t, m_offset));
+      return 0; }
+    '''
+    with tempfile.TemporaryDirectory() as d:
+        src, exe = os.path.join(d, "l.c"), os.path.join(d, "l")
+        open(src, "w").write(prog)
+        subprocess.check_call(["gcc", "-I", os.path.dirname(HEADER), src, "-o", exe])
+        got = [int(x) for x in subprocess.check_output([exe]).split()]
+    want = [C.sizeof(S.ParamDesc), C.sizeof(S.HParams), C.sizeof(S.TensorInfo), S.ParamDesc.shape.offset,
+            S.ParamDesc.ndim.offset, S.ParamDesc.flags.offset, S.TensorInfo.m_offset.offset]
+    assert got == want
+
+
+def _descs(wl, base=0x100000):
+    out = []
+    for k, s in enumerate(wl.specs):
+        shp = (s.shape[0], s.shape[1] if len(s.shape) == 2 else 0)
+        out.append(S.ParamDesc(base * (k + 1), base * (k + 1) + 64, (C.c_int64 * 2)(*shp), len(s.shape), s.tier,
+                               S.F_NO_DECAY if s.no_decay else 0, 0))
+    return out
+
+
+@pytest.mark.parametrize("name", ["toy", "slice", "appb", "literal", "skewed", "ablation"])
+def test_state_bytes_is_closed_form(name):
+    wl = WL.get(name)
+    for policy in (wl.hp.policy, S.POLICY_UNIFORM, S.POLICY_FACTORED_ROUTER):
+        h = S.skew_create(_descs(wl), S.hparams(policy=policy))
+        want = O.state_bytes([(s.shape, s.tier) for s in wl.specs], policy)
+        assert S.skew_state_bytes(h) == want
+        S.skew_destroy(h)
+
+
+def test_appb_headline_state_bytes():
+    h = S.skew_create(_descs(WL.appb()), S.hparams())
+    assert S.skew_state_bytes(h) == 1_380_800_000
+    S.skew_destroy(h)
+
+
+@pytest.mark.parametrize("name", ["toy", "ablation"])
+def test_state_layout_tiles_the_buffer(name):
+    """Every state array has its own range, they do not overlap and they cover the buffer."""
+    wl = WL.get(name)
+    h = S.skew_create(_descs(wl), S.hparams(policy=wl.hp.policy))
+    total = S.skew_state_bytes(h) // 4
+    spans = []
+    for k, s in enumerate(wl.specs):
+        i = S.skew_tensor_info(h, k)
+        kind, mo, dec = O.resolve(len(s.shape), s.tier, wl.hp.policy, s.no_decay)
+        assert (i.kind, i.momentum, i.decay) == (kind, mo, dec)
+        assert i.numel == s.numel
+        for off, cnt in ((i.m_offset, i.numel), (i.v_offset, i.numel), (i.r_offset, i.rows), (i.c_offset, i.cols)):
+            if off >= 0:
+                spans.append((off, off + cnt))
+        assert (i.m_offset >= 0) == bool(mo)
+        assert (i.v_offset >= 0) == (kind == O.KIND_FULL)
+        assert (i.r_offset >= 0) == (i.c_offset >= 0) == (kind == O.KIND_FACTORED)
+    spans.sort()
+    assert spans[0][0] == 0 and spans[-1][1] == total
+    assert all(a[1] == b[0] for a, b in zip(spans, spans[1:]))   # no gap, no overlap
+    S.skew_destroy(h)
+
+
+def _one(shape=(4, 8), tier=S.TIER_EXPERT, **kw):
+    d = dict(weight=0x1000, grad=0x2000, ndim=len(shape), tier=tier, flags=0, reserved=0)
+    d.update(kw)
+    shp = (shape[0], shape[1] if len(shape) == 2 else 0)
+    return S.ParamDesc(d["weight"], d["grad"], (C.c_int64 * 2)(*shp), d["ndim"], d["tier"], d["flags"], d["reserved"])
+
+
+@pytest.mark.parametrize("desc,msg", [
+    (dict(weight=0), "null"), (dict(grad=0), "null"), (dict(weight=0x1001), "aligned"), (dict(ndim=3), "ndim"),
+    (dict(tier=5), "tier"), (dict(flags=8), "flags"), (dict(reserved=1), "reserved"),
+])
+def test_create_rejects_bad_descriptors(desc, msg):
+    with pytest.raises(S.SkewError) as e:
+        S.skew_create([_one(**desc)], S.hparams())
+    assert e.value.code == S.SKEW_EINVAL and msg in str(e.value)
+
+
+@pytest.mark.parametrize("shape", [(0, 8), (8, 0), (-1, 4), (2**41, 2)])
+def test_create_rejects_bad_extents(shape):
+    with pytest.raises(S.SkewError):
+        S.skew_create([_one(shape)], S.hparams())
+
+
+@pytest.mark.parametrize("hp", [dict(beta1=1.0), dict(beta2=-0.1), dict(eps=0.0), dict(eps=float("nan")),
+                                dict(clip_d=0.0), dict(weight_decay=-1.0), dict(policy=7), dict(beta1=float("inf"))])
+def test_create_rejects_bad_hparams(hp):
+    with pytest.raises(S.SkewError) as e:
+        S.skew_create([_one()], S.hparams(**hp))
+    assert e.value.code == S.SKEW_EINVAL
+
+
+def test_step_before_bind_and_bad_bind_sizes():
+    h = S.skew_create([_one()], S.hparams())
+    with pytest.raises(S.SkewError) as e:
+        S.skew_step(h, 1, 1e-3, 0, 0)
+    assert e.value.code == S.SKEW_ESTATE
+    with pytest.raises(S.SkewError) as e:   # wrong sizes are rejected before any CUDA call
+        S.skew_bind(h, 0x100000, S.skew_state_bytes(h) + 4, 0x200000, S.skew_workspace_bytes(h), 0)
+    assert e.value.code == S.SKEW_EINVAL
+    with pytest.raises(S.SkewError) as e:
+        S.skew_bind(h, 0x100010, S.skew_state_bytes(h), 0x200000, S.skew_workspace_bytes(h), 0)
+    assert e.value.code == S.SKEW_EINVAL and "aligned" in str(e.value)
+    with pytest.raises(S.SkewError):
+        S.skew_tensor_info(h, 3)
+    S.skew_destroy(h)
+
+
+def test_empty_parameter_list():
+    h = S.skew_create([], S.hparams())
+    assert S.skew_state_bytes(h) == 0 and S.skew_num_tensors(h) == 0
+    S.skew_destroy(h)
+
+
+def test_64bit_extents_plan():
+    """A tensor past 2^31 elements plans fine (64-bit indexing, cf. the 2^31 crash of 8-bit optimizers)."""
+    h = S.skew_create([_one((65536, 40000)), _one((3 * 2**30,), tier=S.TIER_BACKBONE)], S.hparams())
+    i = S.skew_tensor_info(h, 0)
+    assert i.numel == 65536 * 40000 > 2**31
+    assert S.skew_state_bytes(h) == 4 * (65536 + 40000) + 4 * 2 * 3 * 2**30
+    S.skew_destroy(h)

@@ -1,0 +1,197 @@
+"""GPU parity: libskewadam through its C ABI against the CPU oracle (teacher forced).
+
+Covers the toy MoE set over its 10 steps (zero-grad experts on odd steps, so
+Rbar = 0 at step 1), the paper's own hyper-parameters (eps = 1e-8 clamps at
+step 1), ragged / awkward shapes on the vector and scalar paths, misaligned
+pointers, and the large shape sets at full size in the launch configuration
+the benchmark uses, checking a subset of their tensors.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_19058_gb300 import skewadam as S
+from paper_2607_19058_gb300 import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2607_19058_gb300 import _build
+    _build.build()
+    import oracle
+    oracle.build()
+
+
+def _harness(*a, **k):
+    import parity
+    return parity.Harness(*a, **k)
+
+
+def test_toy_all_steps():
+    h = _harness(WL.toy())
+    for t in range(1, 11):
+        rep = h.step(t)
+        assert rep.tensors == len(h.wl.specs)
+    h.close()
+
+
+def test_toy_paper_hyperparameters():
+    """eps = 1e-8, lr = 3e-4, lambda = 0.05 (App. A): the eps clamp binds at step 1."""
+    h = _harness(WL.toy(), hp_override=dict(eps=1e-8, lr=3e-4, weight_decay=0.05))
+    for t in range(1, 4):
+        h.step(t, seed=77)
+    h.close()
+
+
+def _edge_workload():
+    B, E, R = WL.TIER_BACKBONE, WL.TIER_EXPERT, WL.TIER_ROUTER
+    specs = [WL.Spec("e300x1000", (300, 1000), E), WL.Spec("b517x136", (517, 136), B),
+             WL.Spec("v100003", (100003,), B), WL.Spec("router4096x127", (4096, 127), R),
+             WL.Spec("b1x4096", (1, 4096), B), WL.Spec("e4095x1000", (4095, 1000), E),
+             WL.Spec("e3x5", (3, 5), E), WL.Spec("e7x1", (7, 1), E), WL.Spec("b1x7", (1, 7), B),
+             WL.Spec("v13", (13,), B), WL.Spec("b2x2", (2, 2), B), WL.Spec("e11x13", (11, 13), E),
+             WL.Spec("router8x127", (8, 127), R), WL.Spec("e64x8", (64, 8), E), WL.Spec("e2000x24", (2000, 24), E),
+             WL.Spec("nodecay", (129, 256), B, no_decay=True)]
+    return WL.Workload("edge", specs, WL.HP(), "normal", steps=4)
+
+
+def test_edge_shapes():
+    h = _harness(_edge_workload())
+    for t in range(1, 5):
+        h.step(t, seed=t * 1001)
+    h.close()
+
+
+def test_misaligned_pointers_use_scalar_path():
+    wl = _edge_workload()
+    h = _harness(wl, misalign=(0, 1, 2, 3, 5))
+    for k in (0, 1, 2, 3, 5):
+        assert h.opt.info(k).vectorized == 0
+    assert h.opt.info(4).vectorized == 1
+    for t in range(1, 3):
+        h.step(t, seed=5)
+    h.close()
+
+
+@pytest.mark.parametrize("policy", [WL.POLICY_EXPERT_MOMENTUM, WL.POLICY_FACTORED_ROUTER, WL.POLICY_UNIFORM])
+def test_table3_variants(policy):
+    wl = WL.toy()
+    wl.hp = WL.HP(policy=policy)
+    h = _harness(wl)
+    for t in range(1, 4):
+        h.step(t)
+    h.close()
+
+
+def test_state_bytes_equal_closed_form_and_layout():
+    import oracle as O
+    for name in ("toy", "slice", "appb", "ablation"):
+        wl = WL.get(name)
+        descs = []
+        buf = torch.empty(2, dtype=torch.bfloat16, device="cuda")
+        import ctypes as C
+        for s in wl.specs:
+            shp = (s.shape[0], s.shape[1] if len(s.shape) == 2 else 0)
+            descs.append(S.ParamDesc(buf.data_ptr(), buf.data_ptr(), (C.c_int64 * 2)(*shp), len(s.shape), s.tier, 0, 0))
+        h = S.skew_create(descs, S.hparams(policy=wl.hp.policy))
+        assert S.skew_state_bytes(h) == O.state_bytes([(s.shape, s.tier) for s in wl.specs], wl.hp.policy)
+        S.skew_destroy(h)
+
+
+def test_empty_handle_steps():
+    h = S.skew_create([], S.hparams())
+    assert S.skew_state_bytes(h) == 0
+    ws = torch.empty(max(1, S.skew_workspace_bytes(h)), dtype=torch.uint8, device="cuda")
+    S.skew_bind(h, 0, 0, ws.data_ptr(), S.skew_workspace_bytes(h), torch.cuda.current_stream().cuda_stream)
+    S.skew_step(h, 1, 1e-3, 0, torch.cuda.current_stream().cuda_stream)
+    S.skew_sync_status(h, torch.cuda.current_stream().cuda_stream)
+    S.skew_destroy(h)
+
+
+def test_deterministic_and_resumable():
+    """Same inputs -> bit-identical weights and state; save/restore mid-run changes nothing."""
+    wl = _edge_workload()
+
+    def run(steps, restore_at=None):
+        import parity
+        h = parity.Harness(wl, check=[])
+        snap = None
+        for t in range(1, steps + 1):
+            h.step(t, seed=99)
+            if restore_at == t:
+                snap = ([w.clone() for w in h.W], h.opt.state.clone())
+        if snap is not None:
+            h2 = parity.Harness(wl, check=[])
+            for w, s in zip(h2.W, snap[0]):
+                w.copy_(s)
+            h2.opt.state.copy_(snap[1])
+            for t in range(restore_at + 1, steps + 1):
+                h2.step(t, seed=99)
+            h = h2
+        torch.cuda.synchronize()
+        return [w.clone() for w in h.W], h.opt.state.clone()
+
+    w1, s1 = run(5)
+    w2, s2 = run(5)
+    w3, s3 = run(5, restore_at=2)
+    for a, b, c in zip(w1, w2, w3):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+        assert torch.equal(a.view(torch.int16), c.view(torch.int16))
+    assert torch.equal(s1, s2) and torch.equal(s1, s3)
+
+
+def _subset(wl, names):
+    idx = [k for k, s in enumerate(wl.specs) if s.name in names]
+    assert len(idx) == len(names), names
+    return idx
+
+
+def test_slice_full_size_subset():
+    wl = WL.slice_()
+    chk = _subset(wl, ["attn.q", "attn.k", "norm.attn", "router", "expert0.w0", "expert0.w1", "expert77.w2",
+                       "expert127.w1"])
+    h = _harness(wl, check=chk)
+    for t in (1, 2, 3):
+        h.step(t)
+    h.close()
+
+
+def test_appb_full_size_subset():
+    wl = WL.appb()
+    chk = _subset(wl, ["embed", "pos", "b0.ln1.weight", "b0.attn.k", "b1.attn.o", "b1.router", "expert3.w1",
+                       "expert127.w2", "ln_f.bias"])
+    h = _harness(wl, check=chk)
+    for t in (1, 2):
+        h.step(t)
+    h.close()
+
+
+def test_skewed_full_size_subset():
+    """Zipf loads: 40 zero-grad experts per step, Student-t grads, 100x router spikes at t % 10 == 7."""
+    wl = WL.skewed()
+    ranks = WL.zipf_ranks(wl.n_experts, wl.seed, 7)
+    zero_e = int(np.argmax(ranks.numpy()))          # least loaded at step 7 -> zero grads
+    busy_e = int(np.argmin(ranks.numpy()))
+    chk = _subset(wl, ["b1.router", "b0.attn.q", f"expert{zero_e}.w0", f"expert{busy_e}.w1", "b0.ln2.bias"])
+    h = _harness(wl, check=chk)
+    clipped = 0
+    for t in range(1, 8):
+        if t in (1, 6, 7):
+            rep = h.step(t)
+            clipped += rep.clipped
+        else:
+            h.load_grads(t)
+            h.opt.step(t, h.lr, 1234)
+    assert clipped >= 1
+    h.close()
+
+
+def test_ablation_awkward_full_size_subset():
+    wl = WL.ablation()
+    chk = _subset(wl, ["embed", "odd.a", "odd.b", "b1.router", "expert0.w0", "expert5.w2", "b1.ln2.weight"])
+    h = _harness(wl, check=chk)
+    for t in (1, 2):
+        h.step(t)
+    h.close()
