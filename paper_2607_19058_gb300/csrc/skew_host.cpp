@@ -218,7 +218,7 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
             p.ws_rsum = w; w = align_up(w + 8 * size_t(p.nfr), 256);
         }
         p.ws_u2 = w;
-        w = align_up(w + 4 * size_t(p.ntiles), 256);
+        w = align_up(w + 8 * size_t(p.ntiles), 256);
     }
     h->ws_bytes = w;
     *out = h;
@@ -291,7 +291,7 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.colp = p.kind == kKindFactored ? (float *)(h->ws + p.ws_colp) : nullptr;
         T.bsc = p.kind == kKindFactored ? (float *)(h->ws + p.ws_bsc) : nullptr;
         T.rsum = p.kind == kKindFactored ? (double *)(h->ws + p.ws_rsum) : nullptr;
-        T.u2 = (float *)(h->ws + p.ws_u2);
+        T.u2 = (float2 *)(h->ws + p.ws_u2);
         T.n = p.n;
         T.m = p.m;
         T.numel = p.numel;

@@ -129,6 +129,59 @@ __device__ __forceinline__ float row_scale(float Ri, float rbar_s, int rbar_e) {
     return __frsqrt_rn(__fdiv_rn(ldexpf(Ri, rbar_e), rbar_s));
 }
 
+// Error-free sum (Knuth's TwoSum): s + e == a + b exactly.
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = a + b;
+    const float bp = s - a;
+    e = (a - (s - bp)) + (b - bp);
+}
+
+// Compensated accumulator: the running sum is hi + lo.
+struct Acc2 {
+    float hi = 0.f, lo = 0.f;
+    __device__ __forceinline__ void add(float v) {
+        float s, e;
+        two_sum(hi, v, s, e);
+        hi = s;
+        lo += e;
+    }
+};
+
+// Sum of the squares of eight values by a balanced tree (exact doubling when equal).
+__device__ __forceinline__ float sumsq8(const float (&u)[8]) {
+    const float p01 = fmaf(u[0], u[0], u[1] * u[1]);
+    const float p23 = fmaf(u[2], u[2], u[3] * u[3]);
+    const float p45 = fmaf(u[4], u[4], u[5] * u[5]);
+    const float p67 = fmaf(u[6], u[6], u[7] * u[7]);
+    return (p01 + p23) + (p45 + p67);
+}
+
+// CTA-wide compensated sum of (hi, lo) pairs; result valid in thread 0.
+__device__ float2 block_sum2(Acc2 a, float2 *red) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const float h = __shfl_xor_sync(kAll, a.hi, o), l = __shfl_xor_sync(kAll, a.lo, o);
+        float s, e;
+        two_sum(a.hi, h, s, e);
+        a.hi = s;
+        a.lo += l + e;
+    }
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    __syncthreads();
+    if (l == 0) red[w] = make_float2(a.hi, a.lo);
+    __syncthreads();
+    Acc2 r;
+    if (threadIdx.x == 0) {
+        for (int k = 0; k < kThreads / 32; ++k) {
+            float s, e;
+            two_sum(r.hi, red[k].x, s, e);
+            r.hi = s;
+            r.lo += red[k].y + e;
+        }
+    }
+    return make_float2(r.hi, r.lo);
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(kAll, v, o);
@@ -141,21 +194,7 @@ __device__ __forceinline__ double warp_sum_d(double v) {
     return v;
 }
 
-// Deterministic CTA-wide sums (fixed shuffle tree, then warp 0 over the 8 warp sums).
-__device__ float block_sum(float v, float *red) {
-    v = warp_sum(v);
-    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-    __syncthreads();
-    if (l == 0) red[w] = v;
-    __syncthreads();
-    float r = 0.f;
-    if (w == 0) {
-        r = l < kThreads / 32 ? red[l] : 0.f;
-        r = warp_sum(r);
-    }
-    return r;  // valid in thread 0
-}
-
+// Deterministic CTA-wide fp64 sum (fixed shuffle tree, then warp 0 over the 8 warp sums).
 __device__ double block_sum_d(double v, double *red) {
     v = warp_sum_d(v);
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
@@ -301,7 +340,7 @@ __global__ void __launch_bounds__(kThreads) k_finalize(StepArgs A) {
 // Phase 3: second moment / momentum update and sum(U^2) (Algorithm 1).
 // ---------------------------------------------------------------------------
 template <bool VEC>
-__device__ float rms_fact_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile, float *sm) {
+__device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile, float *sm) {
     const FactTile F(T, tile);
     const uint32_t rt = tile / T.strips;
     for (uint32_t r = threadIdx.x; r < T.tile_rows; r += kThreads) {
@@ -312,7 +351,7 @@ __device__ float rms_fact_tile(const StepArgs &A, const TensorDev &T, const Tens
     float b[8];
     if (F.act)
         load_f8<VEC>(T.bsc + F.col0, F.valid, b);
-    float acc = 0.f;
+    Acc2 acc;
     if (!F.act) return acc;
 #pragma unroll 2
     for (int k = 0; k < kVecPerThread; ++k) {
@@ -329,20 +368,17 @@ __device__ float rms_fact_tile(const StepArgs &A, const TensorDev &T, const Tens
             store_f8<VEC>(T.M + e0, F.valid, y);
         }
         const float a = sm[F.rg + k * F.RG];
+        float u[8];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-            if (c < F.valid) {
-                const float u = y[c] * fminf(a * b[c], A.ce);
-                acc = fmaf(u, u, acc);
-            }
-        }
+        for (int c = 0; c < 8; ++c) u[c] = c < F.valid ? y[c] * fminf(a * b[c], A.ce) : 0.f;
+        acc.add(sumsq8(u));
     }
     return acc;
 }
 
 template <bool VEC>
-__device__ float rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t tile) {
-    float acc = 0.f;
+__device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t tile) {
+    Acc2 acc;
     for (int k = 0; k < kVecPerThread; ++k) {
         const int64_t e0 = 8 * (int64_t(tile) * kThreads * kVecPerThread + int64_t(k) * kThreads + threadIdx.x);
         if (e0 >= T.numel) break;
@@ -363,31 +399,28 @@ __device__ float rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t t
 #pragma unroll
             for (int c = 0; c < 8; ++c) y[c] = g[c];
         }
+        float u[8];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-            if (c < valid) {
-                const float u = y[c] * fminf(__frsqrt_rn(v[c]), A.ce);
-                acc = fmaf(u, u, acc);
-            }
-        }
+        for (int c = 0; c < 8; ++c) u[c] = c < valid ? y[c] * fminf(__frsqrt_rn(v[c]), A.ce) : 0.f;
+        acc.add(sumsq8(u));
     }
     return acc;
 }
 
 __global__ void __launch_bounds__(kThreads) k_rms(StepArgs A) {
     __shared__ float sm[kSmemFloats];
-    __shared__ float red[kThreads / 32];
+    __shared__ float2 red[kThreads / 32];
     __shared__ double redd[kThreads / 32];
     __shared__ int last;
     const uint2 it = A.items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
     TensorScal &S = A.scal[it.x];
-    float acc;
+    Acc2 acc;
     if (T.kind == kKindFactored)
         acc = T.vec ? rms_fact_tile<true>(A, T, S, it.y, sm) : rms_fact_tile<false>(A, T, S, it.y, sm);
     else
         acc = T.vec ? rms_full_tile<true>(A, T, it.y) : rms_full_tile<false>(A, T, it.y);
-    const float tsum = block_sum(acc, red);
+    const float2 tsum = block_sum2(acc, red);
     if (threadIdx.x == 0) {
         T.u2[it.y] = tsum;
         __threadfence();
@@ -399,7 +432,10 @@ __global__ void __launch_bounds__(kThreads) k_rms(StepArgs A) {
     // Last tile of the tensor: sum(U^2), RMS, clip factor (fixed summation order).
     __threadfence();
     double s = 0.0;
-    for (uint32_t k = threadIdx.x; k < T.ntiles; k += kThreads) s += (double)__ldcg(T.u2 + k);
+    for (uint32_t k = threadIdx.x; k < T.ntiles; k += kThreads) {
+        const float2 p = __ldcg(T.u2 + k);
+        s += (double)p.x + (double)p.y;
+    }
     s = block_sum_d(s, redd);
     if (threadIdx.x == 0) {
         const double coef = T.momentum ? A.coef_mom : A.coef_plain;

@@ -29,7 +29,7 @@ struct TensorDev {
     float *colp;        // factored: column partials [rowtiles][m]
     float *bsc;         // factored: 1/sqrt(C_j) [m]
     double *rsum;       // factored: per finalize-row-item sum of R [nfr]
-    float *u2;          // per tile sum of (U / coef)^2 [ntiles]
+    float2 *u2;         // per tile sum of (U / coef)^2 as a (hi, lo) pair [ntiles]
     int64_t n, m, numel;
     uint32_t tid;       // dither tensor id
     uint32_t kind, momentum, decay;
