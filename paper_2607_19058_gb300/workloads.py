@@ -154,7 +154,18 @@ def ablation() -> Workload:
     return Workload("ablation", specs, HP(policy=POLICY_EXPERT_MOMENTUM), "normal", steps=20, n_experts=128)
 
 
-WORKLOADS = {"toy": toy, "slice": slice_, "appb": appb, "literal": literal, "skewed": skewed,
+def small() -> Workload:
+    """A 573M-parameter cut of the App. B set (32 experts, a 4096^2 and a 1024x4096 backbone
+    matrix, 2 norm vectors, the router): 2.3 GB of weights + gradients, well above L2,
+    for profiler captures that must stay small."""
+    d = 4096
+    specs = [Spec("b.q", (d, d), TIER_BACKBONE), Spec("b.k", (1024, d), TIER_BACKBONE)] + _norm("ln", d)
+    specs += [Spec("router", (d, 128), TIER_ROUTER)]
+    specs += _experts(32, [(d, d)])
+    return Workload("small", specs, HP(), "normal", steps=20, n_experts=32)
+
+
+WORKLOADS = {"small": small, "toy": toy, "slice": slice_, "appb": appb, "literal": literal, "skewed": skewed,
              "ablation": ablation}
 
 
