@@ -55,6 +55,7 @@ extern "C" {
 #define SKEW_ECUDA (-3)    /* a CUDA runtime call failed                                   */
 #define SKEW_ETIMEOUT (-4) /* a bounded device-side wait gave up (see skew_sync_status)    */
 #define SKEW_ESTATE (-5)   /* call out of order (e.g. skew_step before skew_bind)          */
+#define SKEW_ETOOBIG (-6)  /* tensor needs more scratch than skew_step_tensor_noalloc has */
 
 /* ---- tiers (Sec. 3 "The tiers") -------------------------------------------- */
 #define SKEW_TIER_BACKBONE 0 /* embeddings, positions, attention, dense FFN, norms */
@@ -218,6 +219,46 @@ int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *ou
 int skew_profile_begin(skew_handle_t *h, int32_t max_steps);
 int skew_profile_end(skew_handle_t *h, double *ms, int64_t cap, int32_t *n_steps, int32_t *n_kernels);
 const char *skew_kernel_name(int32_t k);
+
+/*
+ * A step over ONE tensor that allocates nothing -- no cudaMalloc / cudaFree, no
+ * allocating library routine, no host heap. The paper has no counterpart; this
+ * is a deployment convenience.
+ *
+ * Who needs it: callers that cannot allocate device memory when they step the
+ * optimizer, e.g. code running while a framework's caching allocator holds all
+ * free memory, plugins that are only handed pre-sized buffers, or runtimes that
+ * forbid allocation after start-up. skew_bind needs a caller-allocated
+ * workspace; this entry point instead uses a fixed scratch array compiled into
+ * the library: SKEW_NOALLOC_SCRATCH_BYTES of device memory on every GPU that
+ * loads the library, held until the process exits. That is enough for one
+ * tensor of up to about 50,000 x 4,096 (the paper's 50,304 x 4,096 embedding
+ * fits); larger tensors are rejected with SKEW_ETOOBIG before any work is
+ * enqueued.
+ *
+ * Arguments: weight / grad as in skew_param_desc_t (device, bf16, row-major);
+ * ndim, rows, cols, tier, flags as in skew_param_desc_t; hp as for
+ * skew_create; state: this tensor's fp32 state, exactly state_bytes =
+ * 4 * ((momentum ? numel : 0) + (full second moment ? numel : rows + cols))
+ * bytes, laid out [M][v] or [M][R][C] (absent arrays take no room), 4-byte
+ * aligned, zero-filled by the caller before the first step; tensor_id: the id
+ * fed to the dither (use the tensor's index in a skew_create list to get the
+ * same bits as skew_step); step, lr, seed as for skew_step; stream: a
+ * cudaStream_t. Updates weight and state in place, asynchronously on stream,
+ * with the same kernels and results as skew_step on a one-tensor handle.
+ *
+ * The first call on a device looks up the array's device address with
+ * cudaGetSymbolAddress (with that device current); make that first call before
+ * any stream capture. All calls on a device share the one array: calls whose
+ * work overlaps on the GPU (different streams, or other host threads) race
+ * and corrupt each other's results -- serialise them. The array keeps the
+ * last call's contents; everything a step needs zeroed is cleared by the step.
+ * Errors: SKEW_EINVAL (argument or state size), SKEW_ETOOBIG, SKEW_ECUDA.
+ */
+#define SKEW_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t ndim, int64_t rows, int64_t cols, int32_t tier,
+                             uint32_t flags, const skew_hparams_t *hp, void *state, size_t state_bytes,
+                             uint32_t tensor_id, int64_t step, float lr, uint64_t seed, void *stream);
 
 /* Number of tensors the handle plans for (0 for NULL). */
 int32_t skew_num_tensors(const skew_handle_t *h);

@@ -13,7 +13,7 @@ OBJ = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libskewadam.so")
 INCLUDE = os.path.join(ROOT, "include")
 
-SOURCES = ["skew_host.cpp", "skew_kernels.cu"]
+SOURCES = ["skew_host.cpp", "skew_kernels.cu", "skew_noalloc.cu"]
 HEADERS = [os.path.join(CSRC, "skew_plan.h"), os.path.join(INCLUDE, "skewadam.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",

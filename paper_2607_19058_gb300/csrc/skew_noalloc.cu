@@ -1,0 +1,232 @@
+// skew_step_tensor_noalloc: a SkewAdam step over one tensor that allocates nothing.
+//
+// The regular path (skew_create / skew_bind / skew_step) needs a caller-allocated
+// workspace for its scratch: row / column partial sums, per-tile sums of U^2,
+// per-tensor scalars and the tile tables. Some callers cannot allocate device
+// memory at the point where they step the optimizer -- for example code that
+// runs while a framework's caching allocator owns every free byte, plugins that
+// are handed only pre-sized buffers, or runtimes that forbid cudaMalloc after
+// start-up. For them this entry point keeps the scratch in a fixed array
+// compiled into the library (g_scratch below, SKEW_NOALLOC_SCRATCH_BYTES bytes
+// in the device memory of every GPU that loads the library, held until the
+// process exits) and launches the same four kernels as skew_step.
+//
+// The array's address is a device address that host code cannot name
+// directly: the host-side symbol is only a stand-in. It is looked up once per
+// device with cudaGetSymbolAddress, with that device current, on the first
+// call made on that device.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <mutex>
+
+#include "skew_plan.h"
+#include "skewadam.h"
+
+namespace skew {
+namespace {
+
+static __device__ __align__(256) unsigned char g_scratch[SKEW_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+unsigned char *g_scratch_ptr[kMaxDevices] = {};
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Writes the descriptor, clears the scalars (the step's completion counters
+// must start at zero) and fills the three item tables of one tensor.
+__global__ void k_noalloc_setup(TensorDev td, TensorDev *dst, TensorScal *scal, uint32_t *err, uint2 *itemsA,
+                                uint32_t nA, uint2 *itemsF, uint32_t nF, uint2 *itemsBC, uint32_t nBC) {
+    const uint32_t stride = gridDim.x * blockDim.x;
+    const uint32_t i0 = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i0 == 0) {
+        *dst = td;
+        *scal = TensorScal{};
+        *err = 0;
+    }
+    for (uint32_t i = i0; i < nA; i += stride) itemsA[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < nF; i += stride) itemsF[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < nBC; i += stride) itemsBC[i] = make_uint2(0, i);
+}
+
+}  // namespace
+}  // namespace skew
+
+using namespace skew;
+
+extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t ndim, int64_t rows, int64_t cols,
+                                        int32_t tier, uint32_t flags, const skew_hparams_t *hp, void *state,
+                                        size_t state_bytes, uint32_t tensor_id, int64_t step, float lr, uint64_t seed,
+                                        void *stream) {
+    // ---- arguments (same rules as skew_create / skew_step) ------------------
+    if (!hp || !weight || !grad || !state) return SKEW_EINVAL;
+    if (((uintptr_t)weight & 1) || ((uintptr_t)grad & 1)) return SKEW_EINVAL;
+    if (((uintptr_t)state & 3)) return SKEW_EINVAL;
+    if (ndim != 1 && ndim != 2) return SKEW_EINVAL;
+    if (tier < SKEW_TIER_BACKBONE || tier > SKEW_TIER_ROUTER) return SKEW_EINVAL;
+    if (flags & ~SKEW_F_NO_DECAY) return SKEW_EINVAL;
+    const skew_hparams_t H = *hp;
+    if (!std::isfinite(H.beta1) || H.beta1 < 0.f || H.beta1 >= 1.f) return SKEW_EINVAL;
+    if (!std::isfinite(H.beta2) || H.beta2 < 0.f || H.beta2 >= 1.f) return SKEW_EINVAL;
+    if (!std::isfinite(H.eps) || !(H.eps > 0.f)) return SKEW_EINVAL;
+    if (!std::isfinite(H.clip_d) || !(H.clip_d > 0.f)) return SKEW_EINVAL;
+    if (!std::isfinite(H.weight_decay) || H.weight_decay < 0.f) return SKEW_EINVAL;
+    if (H.policy < SKEW_POLICY_TIERED || H.policy > SKEW_POLICY_UNIFORM) return SKEW_EINVAL;
+    if (step < 1) return SKEW_EINVAL;
+    if (!std::isfinite(lr) || lr < 0.f) return SKEW_EINVAL;
+    const int64_t n = rows, m = ndim == 2 ? cols : 1;
+    if (n < 1 || m < 1 || n > (int64_t(1) << 40) || m > (int64_t(1) << 40) || n > (int64_t(1) << 62) / m)
+        return SKEW_EINVAL;
+    const int64_t numel = n * m;
+
+    // ---- tier policy (as the planner's, Sec. 3 "The tiers" / Table 3) -------------
+    uint32_t kind, momentum, decay;
+    if (ndim == 1 || (tier == SKEW_TIER_ROUTER && H.policy != SKEW_POLICY_FACTORED_ROUTER && H.policy != SKEW_POLICY_UNIFORM))
+        kind = kKindFull;
+    else
+        kind = kKindFactored;
+    if (tier == SKEW_TIER_BACKBONE)
+        momentum = 1;
+    else if (tier == SKEW_TIER_EXPERT)
+        momentum = (H.policy == SKEW_POLICY_EXPERT_MOMENTUM || H.policy == SKEW_POLICY_UNIFORM);
+    else
+        momentum = (H.policy == SKEW_POLICY_UNIFORM);
+    decay = (tier != SKEW_TIER_ROUTER) && !(flags & SKEW_F_NO_DECAY);
+
+    // ---- caller's state: [M][v][R][C] of this tensor, exactly the closed form -----
+    const int64_t state_floats = (momentum ? numel : 0) + (kind == kKindFull ? numel : n + m);
+    if (state_bytes != size_t(state_floats) * 4) return SKEW_EINVAL;
+    float *sf = reinterpret_cast<float *>(state);
+    float *M = momentum ? sf : nullptr;
+    float *after_m = sf + (momentum ? numel : 0);
+    float *v = kind == kKindFull ? after_m : nullptr;
+    float *R = kind == kKindFactored ? after_m : nullptr;
+    float *Cc = kind == kKindFactored ? after_m + n : nullptr;
+
+    // ---- tile geometry (the planner's: 8-element vectors, 16 rows per thread) -------
+    uint32_t lcl = 0, strips = 1, rowtiles, tile_rows = 0, ntiles, nfr = 0, nfc = 0;
+    if (kind == kKindFactored) {
+        const int64_t vecs = (m + 7) / 8;
+        uint32_t lc = 1;
+        while (lc < 32 && lc < vecs) {
+            lc <<= 1;
+            ++lcl;
+        }
+        strips = (uint32_t)((m + 8 * lc - 1) / (8 * lc));
+        tile_rows = (uint32_t)(kVecPerThread * (kThreads / lc));
+        rowtiles = (uint32_t)((n + tile_rows - 1) / tile_rows);
+        nfr = (uint32_t)((n + kFinChunk - 1) / kFinChunk);
+        nfc = (uint32_t)((m + kFinChunk - 1) / kFinChunk);
+    } else {
+        rowtiles = (uint32_t)((numel + kFlatTileElems - 1) / kFlatTileElems);
+    }
+    ntiles = strips * rowtiles;
+    const uint32_t nA = kind == kKindFactored ? ntiles : 0, nF = nfr + nfc, nBC = ntiles;
+
+    // ---- scratch layout inside the fixed array --------------------------------------
+    size_t off = 0;
+    const size_t o_scal = off;   off = align256(off + sizeof(TensorScal));
+    const size_t o_err = off;    off = align256(off + 16);
+    const size_t o_tens = off;   off = align256(off + sizeof(TensorDev));
+    const size_t o_iA = off;     off = align256(off + sizeof(uint2) * nA);
+    const size_t o_iF = off;     off = align256(off + sizeof(uint2) * nF);
+    const size_t o_iBC = off;    off = align256(off + sizeof(uint2) * nBC);
+    size_t o_rowp = 0, o_colp = 0, o_bsc = 0, o_rsum = 0;
+    if (kind == kKindFactored) {
+        o_rowp = off; off = align256(off + 4 * size_t(strips) * n);
+        o_colp = off; off = align256(off + 4 * size_t(rowtiles) * m);
+        o_bsc = off;  off = align256(off + 4 * size_t(m));
+        o_rsum = off; off = align256(off + 8 * size_t(nfr));
+    }
+    const size_t o_u2 = off;     off = align256(off + 8 * size_t(ntiles));
+    if (off > SKEW_NOALLOC_SCRATCH_BYTES) return SKEW_ETOOBIG;  // too large for the fixed array
+
+    // ---- device address of the fixed array, once per device ------------------------
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return SKEW_ECUDA;
+    if (dev < 0 || dev >= kMaxDevices) return SKEW_EINVAL;
+    unsigned char *base;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        if (!g_scratch_ptr[dev]) {
+            void *p = nullptr;
+            e = cudaGetSymbolAddress(&p, g_scratch);
+            if (e != cudaSuccess || !p) return SKEW_ECUDA;  // the array's device address is unknown
+            g_scratch_ptr[dev] = static_cast<unsigned char *>(p);
+        }
+        base = g_scratch_ptr[dev];
+    }
+
+    TensorDev td{};
+    td.w = (uint16_t *)weight;
+    td.g = (const uint16_t *)grad;
+    td.M = M;
+    td.v = v;
+    td.R = R;
+    td.C = Cc;
+    td.rowp = kind == kKindFactored ? (float *)(base + o_rowp) : nullptr;
+    td.colp = kind == kKindFactored ? (float *)(base + o_colp) : nullptr;
+    td.bsc = kind == kKindFactored ? (float *)(base + o_bsc) : nullptr;
+    td.rsum = kind == kKindFactored ? (double *)(base + o_rsum) : nullptr;
+    td.u2 = (float2 *)(base + o_u2);
+    td.n = n;
+    td.m = m;
+    td.numel = numel;
+    td.tid = tensor_id;
+    td.kind = kind;
+    td.momentum = momentum;
+    td.decay = decay;
+    auto al16 = [](const void *p) { return ((uintptr_t)p & 15) == 0; };
+    bool vec = al16(td.w) && al16(td.g) && (!td.M || al16(td.M));
+    vec = kind == kKindFull ? (vec && numel % 8 == 0 && al16(td.v)) : (vec && m % 8 == 0);
+    td.vec = vec ? 1 : 0;
+    td.lcl = lcl;
+    td.strips = strips;
+    td.rowtiles = rowtiles;
+    td.tile_rows = tile_rows;
+    td.ntiles = ntiles;
+    td.nfr = nfr;
+    td.nfc = nfc;
+
+    cudaStream_t s = (cudaStream_t)stream;
+    k_noalloc_setup<<<8, 256, 0, s>>>(td, (TensorDev *)(base + o_tens), (TensorScal *)(base + o_scal),
+                                      (uint32_t *)(base + o_err), (uint2 *)(base + o_iA), nA, (uint2 *)(base + o_iF),
+                                      nF, (uint2 *)(base + o_iBC), nBC);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return SKEW_ECUDA;
+
+    // ---- per-step scalars, as skew_step forms them ------------------------------------
+    const double t = (double)step;
+    const double bc1 = 1.0 - std::pow((double)H.beta1, t);
+    const double s2 = std::sqrt(1.0 - std::pow((double)H.beta2, t));
+    StepArgs a{};
+    a.tensors = (const TensorDev *)(base + o_tens);
+    a.scal = (TensorScal *)(base + o_scal);
+    a.err = (uint32_t *)(base + o_err);
+    a.b1 = H.beta1;
+    a.b2 = H.beta2;
+    a.c1 = (float)(1.0 - (double)H.beta1);
+    a.c2 = (float)(1.0 - (double)H.beta2);
+    a.ce = (float)(1.0 / std::sqrt((double)H.eps));
+    a.wdf = (float)(1.0 - (double)lr * (double)H.weight_decay);
+    a.lr = lr;
+    a.clip_d = H.clip_d;
+    a.coef_mom = s2 / bc1;
+    a.coef_plain = s2;
+    a.step_lo = (uint32_t)(uint64_t)step;
+    a.seed_lo = (uint32_t)seed;
+    a.seed_hi = (uint32_t)(seed >> 32);
+
+    LaunchPlan lp{};
+    lp.nA = nA;
+    lp.nF = nF;
+    lp.nBC = nBC;
+    lp.itemsA = (const uint2 *)(base + o_iA);
+    lp.itemsF = (const uint2 *)(base + o_iF);
+    lp.itemsBC = (const uint2 *)(base + o_iBC);
+    lp.events = nullptr;
+    e = (cudaError_t)launch_step(lp, a, stream);
+    if (e != cudaSuccess) return SKEW_ECUDA;
+    return SKEW_OK;
+}

@@ -18,7 +18,8 @@ from typing import Iterable, List, Optional, Sequence
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libskewadam.so")
 
-SKEW_OK, SKEW_EINVAL, SKEW_ENOMEM, SKEW_ECUDA, SKEW_ETIMEOUT, SKEW_ESTATE = 0, -1, -2, -3, -4, -5
+SKEW_OK, SKEW_EINVAL, SKEW_ENOMEM, SKEW_ECUDA, SKEW_ETIMEOUT, SKEW_ESTATE, SKEW_ETOOBIG = 0, -1, -2, -3, -4, -5, -6
+NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 TIER_BACKBONE, TIER_EXPERT, TIER_ROUTER = 0, 1, 2
 POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM = 0, 1, 2, 3
 F_NO_DECAY = 1
@@ -26,7 +27,7 @@ KIND_FULL, KIND_FACTORED = 0, 1
 
 EXPORTS = ["skew_create", "skew_destroy", "skew_state_bytes", "skew_workspace_bytes", "skew_bind", "skew_step",
            "skew_sync_status", "skew_tensor_scalars", "skew_tensor_info", "skew_num_tensors", "skew_last_error",
-           "skew_profile_begin", "skew_profile_end", "skew_kernel_name"]
+           "skew_profile_begin", "skew_profile_end", "skew_kernel_name", "skew_step_tensor_noalloc"]
 
 
 class SkewError(RuntimeError):
@@ -95,6 +96,9 @@ def load(path: Optional[str] = None) -> C.CDLL:
         L.skew_profile_end.restype = C.c_int
         L.skew_kernel_name.argtypes = [i32]
         L.skew_kernel_name.restype = C.c_char_p
+        L.skew_step_tensor_noalloc.argtypes = [vp, vp, i32, i64, i64, i32, C.c_uint32, C.POINTER(HParams), vp, sz,
+                                               C.c_uint32, i64, C.c_float, u64, vp]
+        L.skew_step_tensor_noalloc.restype = C.c_int
         if path is None:
             _lib = L
         return L
@@ -178,6 +182,18 @@ def skew_profile_end(h, cap: int = 1 << 16):
 def skew_kernel_name(k: int) -> str:
     m = load().skew_kernel_name(k)
     return m.decode() if m else ""
+
+
+def skew_step_tensor_noalloc(weight_ptr: int, grad_ptr: int, ndim: int, rows: int, cols: int, tier: int, flags: int,
+                             hp: HParams, state_ptr: int, state_bytes: int, tensor_id: int, step: int, lr: float,
+                             seed: int, stream: int) -> None:
+    """One tensor's step with the library's fixed scratch array (no allocation of any kind)."""
+    rc = load().skew_step_tensor_noalloc(weight_ptr, grad_ptr, ndim, rows, cols, tier, flags, C.byref(hp), state_ptr,
+                                         state_bytes, tensor_id, step, lr, seed & (2**64 - 1), stream)
+    if rc != SKEW_OK:
+        why = {SKEW_EINVAL: "invalid argument or state size", SKEW_ECUDA: "CUDA error",
+               SKEW_ETOOBIG: f"tensor needs more than the {NOALLOC_SCRATCH_BYTES} bytes of fixed scratch"}
+        raise SkewError(rc, why.get(rc, "error"))
 
 
 def hparams(beta1=0.9, beta2=0.999, eps=1e-8, clip_d=1.0, weight_decay=0.05, policy=POLICY_TIERED) -> HParams:
