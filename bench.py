@@ -136,6 +136,7 @@ def byte_model(opt, n_tensors):
             rc += i.rows + i.cols
     step_min = 6 * N + 8 * N_mom + 8 * N_full + 8 * rc
     kernels = {
+        "step_graph": step_min,                                  # the whole step: one graph launch
         "k_sumsq": 2 * N_fact,                                   # read G of factored matrices
         "k_finalize": 8 * rc,                                    # R, C read + write
         "k_rms": 2 * N + 8 * N_mom + 8 * N_full,                 # read G; M, v read + write
@@ -379,7 +380,7 @@ def run_ours(args):
             "kernels_ms": kmean,
             "e2e": e2e,
             "cpu_baseline": cpu,
-            "gpu_launches": args.steps * len(names),
+            "gpu_launches": args.steps * S.skew_launches_per_step(opt.h),
             "clocks": clocks,
         }
         print(json.dumps(out))

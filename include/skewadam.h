@@ -208,13 +208,14 @@ int skew_tensor_scalars(skew_handle_t *h, int32_t tid, double out[4], void *stre
 int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *out);
 
 /*
- * Benchmark support: per-kernel timing. After skew_profile_begin(h, n), each of
- * the next n calls of skew_step records a CUDA event before and after every
- * kernel it launches (on the step's stream; no extra synchronisation).
- * skew_profile_end(h, ms, cap, &steps, &kernels) synchronises, writes the
- * durations in milliseconds row-major into ms[steps][kernels] (up to cap
- * values), releases the events and stops recording. skew_kernel_name(k) names
- * kernel k of a step. Errors: SKEW_EINVAL, SKEW_ECUDA.
+ * Benchmark support: launch timing. After skew_profile_begin(h, n), each of the
+ * next n calls of skew_step records a CUDA event before and after each timed
+ * launch it makes on the step's stream (one: the step graph; no extra
+ * synchronisation). skew_profile_end(h, ms, cap, &steps, &launches)
+ * synchronises, writes the durations in milliseconds row-major into
+ * ms[steps][launches] (up to cap values), releases the events and stops
+ * recording. skew_kernel_name(k) names timed launch k of a step.
+ * Errors: SKEW_EINVAL, SKEW_ECUDA.
  */
 int skew_profile_begin(skew_handle_t *h, int32_t max_steps);
 int skew_profile_end(skew_handle_t *h, double *ms, int64_t cap, int32_t *n_steps, int32_t *n_kernels);
@@ -259,6 +260,12 @@ const char *skew_kernel_name(int32_t k);
 int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t ndim, int64_t rows, int64_t cols, int32_t tier,
                              uint32_t flags, const skew_hparams_t *hp, void *state, size_t state_bytes,
                              uint32_t tensor_id, int64_t step, float lr, uint64_t seed, void *stream);
+
+/*
+ * Kernel launches one skew_step performs (the step runs as one captured CUDA
+ * graph of grouped launches; 0 for NULL or an empty handle).
+ */
+int64_t skew_launches_per_step(const skew_handle_t *h);
 
 /* Number of tensors the handle plans for (0 for NULL). */
 int32_t skew_num_tensors(const skew_handle_t *h);

@@ -14,6 +14,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <string>
@@ -35,6 +36,23 @@ thread_local std::string g_create_err;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Integer tuning override from the environment (benchmarking knobs), else `dflt`.
+long env_long(const char *name, long dflt, long lo, long hi) {
+    const char *v = std::getenv(name);
+    if (!v || !*v) return dflt;
+    char *end = nullptr;
+    const long x = std::strtol(v, &end, 10);
+    return (end && *end == 0 && x >= lo && x <= hi) ? x : dflt;
+}
+
+// A unit is a run of consecutive tensors whose phases form one chain of the
+// step graph; its items are ranges of the per-phase item tables.
+struct Unit {
+    uint32_t a0, nA, f0, nF, b0, nBC;
+};
+
+constexpr int kMaxBranches = 8;
+
 }  // namespace
 
 struct skew_handle {
@@ -42,19 +60,42 @@ struct skew_handle {
     skew_hparams_t hp{};
     std::vector<TPlan> t;
     size_t state_bytes = 0, ws_bytes = 0;
-    size_t ws_scal = 0, ws_err = 0, ws_tab = 0, ws_tab_end = 0;
+    size_t ws_scal = 0, ws_err = 0, ws_params = 0, ws_tab = 0, ws_tab_end = 0;
     size_t ws_tens = 0, ws_itemsA = 0, ws_itemsF = 0, ws_itemsBC = 0;
-    std::vector<uint2> itemsA, itemsF, itemsBC;
+    std::vector<uint2> itemsA, itemsF, itemsBC;  // unit by unit, tensors in order
+    std::vector<Unit> units;
+    int branches = 3;
     char *state = nullptr, *ws = nullptr;
     bool bound = false;
     std::string err;
-    // per-kernel timing (skew_profile_begin / skew_profile_end)
+    // the captured step: units round-robin over `branches` streams
+    cudaStream_t br[kMaxBranches] = {};
+    cudaEvent_t fork = nullptr, join[kMaxBranches] = {};
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    // per-launch timing (skew_profile_begin / skew_profile_end)
     std::vector<cudaEvent_t> prof_ev;
     int32_t prof_max = 0, prof_used = 0;
+    void release_graph() {
+        if (exec) cudaGraphExecDestroy(exec);
+        if (graph) cudaGraphDestroy(graph);
+        exec = nullptr;
+        graph = nullptr;
+    }
     ~skew_handle() {
+        release_graph();
+        for (cudaStream_t x : br)
+            if (x) cudaStreamDestroy(x);
+        if (fork) cudaEventDestroy(fork);
+        for (cudaEvent_t e : join)
+            if (e) cudaEventDestroy(e);
         for (cudaEvent_t e : prof_ev) cudaEventDestroy(e);
     }
 };
+
+// What the profiler times per step: the one graph launch.
+constexpr int kProfLaunches = 1;
+const char *const kProfNames[kProfLaunches] = {"step_graph"};
 
 static int fail(skew_handle_t *h, int code, const char *fmt, ...) {
     char buf[512];
@@ -179,15 +220,32 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
         if (p.kind == kKindFactored) { p.coff = off; off += p.m; }
     h->state_bytes = size_t(off) * 4;
 
-    // Work items of the three phases.
+    // Units: consecutive tensors with at least `min_tiles` update tiles (the last
+    // may have fewer), so that one expert matrix is a unit and small tensors are
+    // grouped. Each unit's phases are one chain A -> F -> B -> C of the step graph.
     try {
-        for (int32_t k = 0; k < n_params; ++k) {
-            const TPlan &p = h->t[k];
-            if (p.kind == kKindFactored) {
-                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(k, i));
-                for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(k, i));
+        const long min_tiles = env_long("SKEW_UNIT_MIN_TILES", 1L << 30, 1, 1L << 30);
+        h->branches = (int)env_long("SKEW_BRANCHES", 1, 1, kMaxBranches);
+        int b = 0;
+        long acc = 0;
+        for (int k = 0; k < n_params; ++k) {
+            acc += h->t[k].ntiles;
+            if (acc < min_tiles && k != n_params - 1) continue;
+            Unit u{(uint32_t)h->itemsA.size(), 0, (uint32_t)h->itemsF.size(), 0, (uint32_t)h->itemsBC.size(), 0};
+            for (int q = b; q <= k; ++q) {
+                const TPlan &p = h->t[q];
+                if (p.kind == kKindFactored) {
+                    for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(q, i));
+                    for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(q, i));
+                }
+                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsBC.push_back(make_uint2(q, i));
             }
-            for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsBC.push_back(make_uint2(k, i));
+            u.nA = (uint32_t)h->itemsA.size() - u.a0;
+            u.nF = (uint32_t)h->itemsF.size() - u.f0;
+            u.nBC = (uint32_t)h->itemsBC.size() - u.b0;
+            h->units.push_back(u);
+            b = k + 1;
+            acc = 0;
         }
     } catch (...) {
         delete h;
@@ -200,6 +258,8 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     w = align_up(w + sizeof(TensorScal) * n_params, 256);
     h->ws_err = w;
     w = align_up(w + 16, 256);
+    h->ws_params = w;
+    w = align_up(w + sizeof(StepArgs), 256);
     h->ws_tab = w;
     h->ws_tens = w;
     w = align_up(w + sizeof(TensorDev) * n_params, 256);
@@ -235,6 +295,13 @@ size_t skew_state_bytes(const skew_handle_t *h) { return h ? h->state_bytes : 0;
 size_t skew_workspace_bytes(const skew_handle_t *h) { return h ? h->ws_bytes : 0; }
 
 int32_t skew_num_tensors(const skew_handle_t *h) { return h ? (int32_t)h->t.size() : 0; }
+
+int64_t skew_launches_per_step(const skew_handle_t *h) {
+    if (!h) return 0;
+    int64_t n = 0;
+    for (const Unit &u : h->units) n += (u.nA > 0) + (u.nF > 0) + 2 * (u.nBC > 0);
+    return n;
+}
 
 const char *skew_last_error(const skew_handle_t *h) { return h ? h->err.c_str() : g_create_err.c_str(); }
 
@@ -337,6 +404,44 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         e = cudaMemsetAsync(h->ws + h->ws_scal, 0, h->ws_tab - h->ws_scal, s);
         if (e != cudaSuccess) return cuda_fail(h, e, "zero-fill of the scalars");
     }
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "bind");
+
+    // Capture the step graph: units round-robin over the branch streams, each a
+    // chain A -> F -> B -> C; the branches fork from and join back to branch 0.
+    h->release_graph();
+    if (!h->units.empty()) {
+        for (int b = 0; b < h->branches; ++b) {
+            if (!h->br[b] && (e = cudaStreamCreateWithFlags(&h->br[b], cudaStreamNonBlocking)) != cudaSuccess)
+                return cuda_fail(h, e, "stream create");
+            if (!h->join[b] && (e = cudaEventCreateWithFlags(&h->join[b], cudaEventDisableTiming)) != cudaSuccess)
+                return cuda_fail(h, e, "event create");
+        }
+        if (!h->fork && (e = cudaEventCreateWithFlags(&h->fork, cudaEventDisableTiming)) != cudaSuccess)
+            return cuda_fail(h, e, "event create");
+        const StepArgs *P = reinterpret_cast<const StepArgs *>(h->ws + h->ws_params);
+        const uint2 *iA = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsA);
+        const uint2 *iF = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsF);
+        const uint2 *iBC = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsBC);
+        e = cudaStreamBeginCapture(h->br[0], cudaStreamCaptureModeThreadLocal);
+        if (e != cudaSuccess) return cuda_fail(h, e, "graph capture");
+        cudaError_t ce = cudaEventRecord(h->fork, h->br[0]);
+        for (int b = 1; b < h->branches && ce == cudaSuccess; ++b) ce = cudaStreamWaitEvent(h->br[b], h->fork, 0);
+        for (size_t u = 0; u < h->units.size() && ce == cudaSuccess; ++u) {
+            const Unit &U = h->units[u];
+            const LaunchPlan L{U.nA, U.nF, U.nBC, iA + U.a0, iF + U.f0, iBC + U.b0};
+            ce = (cudaError_t)launch_phases(P, L, h->br[u % h->branches]);
+        }
+        for (int b = 1; b < h->branches && ce == cudaSuccess; ++b) {
+            ce = cudaEventRecord(h->join[b], h->br[b]);
+            if (ce == cudaSuccess) ce = cudaStreamWaitEvent(h->br[0], h->join[b], 0);
+        }
+        e = cudaStreamEndCapture(h->br[0], &h->graph);
+        if (ce != cudaSuccess) return cuda_fail(h, ce, "graph capture");
+        if (e != cudaSuccess) return cuda_fail(h, e, "graph capture");
+        e = cudaGraphInstantiate(&h->exec, h->graph, 0);
+        if (e != cudaSuccess) return cuda_fail(h, e, "graph instantiate");
+    }
     h->bound = true;
     return SKEW_OK;
 }
@@ -356,7 +461,6 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
     StepArgs a{};
     a.tensors = reinterpret_cast<const TensorDev *>(h->ws + h->ws_tens);
     a.scal = reinterpret_cast<TensorScal *>(h->ws + h->ws_scal);
-    a.err = reinterpret_cast<uint32_t *>(h->ws + h->ws_err);
     a.b1 = H.beta1;
     a.b2 = H.beta2;
     a.c1 = (float)(1.0 - (double)H.beta1);
@@ -371,22 +475,21 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
     a.seed_lo = (uint32_t)seed;
     a.seed_hi = (uint32_t)(seed >> 32);
 
-    LaunchPlan lp{};
-    lp.nA = (uint32_t)h->itemsA.size();
-    lp.nF = (uint32_t)h->itemsF.size();
-    lp.nBC = (uint32_t)h->itemsBC.size();
-    lp.itemsA = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsA);
-    lp.itemsF = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsF);
-    lp.itemsBC = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsBC);
-
+    cudaEvent_t *ev = nullptr;
     if (h->prof_used < h->prof_max) {
-        lp.events = reinterpret_cast<void *const *>(h->prof_ev.data() + size_t(h->prof_used) * (kNumKernels + 1));
+        ev = h->prof_ev.data() + size_t(h->prof_used) * (kProfLaunches + 1);
         ++h->prof_used;
     }
-    cudaError_t e = cudaMemsetAsync(h->ws + h->ws_scal, 0, sizeof(TensorScal) * h->t.size(), s);
+    // The parameter block: the copy from this pageable struct is staged before
+    // cudaMemcpyAsync returns, so the struct may go out of scope.
+    cudaError_t e = cudaMemcpyAsync(h->ws + h->ws_params, &a, sizeof a, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "parameter upload");
+    e = cudaMemsetAsync(h->ws + h->ws_scal, 0, sizeof(TensorScal) * h->t.size(), s);
     if (e != cudaSuccess) return cuda_fail(h, e, "reset of per-step scalars");
-    e = (cudaError_t)launch_step(lp, a, stream);
-    if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
+    if (ev) cudaEventRecord(ev[0], s);
+    e = cudaGraphLaunch(h->exec, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "graph launch");
+    if (ev) cudaEventRecord(ev[1], s);
     return SKEW_OK;
 }
 
@@ -396,7 +499,7 @@ int skew_profile_begin(skew_handle_t *h, int32_t max_steps) {
     h->prof_ev.clear();
     h->prof_max = h->prof_used = 0;
     try {
-        h->prof_ev.resize(size_t(max_steps) * (kNumKernels + 1), nullptr);
+        h->prof_ev.resize(size_t(max_steps) * (kProfLaunches + 1), nullptr);
     } catch (...) {
         return fail(h, SKEW_ENOMEM, "out of host memory");
     }
@@ -416,8 +519,8 @@ int skew_profile_end(skew_handle_t *h, double *ms, int64_t cap, int32_t *n_steps
     int rc = SKEW_OK;
     int64_t w = 0;
     for (int32_t st = 0; st < h->prof_used; ++st) {
-        cudaEvent_t *ev = h->prof_ev.data() + size_t(st) * (kNumKernels + 1);
-        for (int k = 0; k < kNumKernels; ++k) {
+        cudaEvent_t *ev = h->prof_ev.data() + size_t(st) * (kProfLaunches + 1);
+        for (int k = 0; k < kProfLaunches; ++k) {
             float t = 0.f;
             cudaError_t e = cudaEventSynchronize(ev[k + 1]);
             if (e == cudaSuccess) e = cudaEventElapsedTime(&t, ev[k], ev[k + 1]);
@@ -427,14 +530,14 @@ int skew_profile_end(skew_handle_t *h, double *ms, int64_t cap, int32_t *n_steps
         }
     }
     if (n_steps) *n_steps = h->prof_used;
-    if (n_kernels) *n_kernels = kNumKernels;
+    if (n_kernels) *n_kernels = kProfLaunches;
     for (cudaEvent_t e : h->prof_ev) cudaEventDestroy(e);
     h->prof_ev.clear();
     h->prof_max = h->prof_used = 0;
     return rc;
 }
 
-const char *skew_kernel_name(int32_t k) { return (k >= 0 && k < kNumKernels) ? kKernelNames[k] : ""; }
+const char *skew_kernel_name(int32_t k) { return (k >= 0 && k < kProfLaunches) ? kProfNames[k] : ""; }
 
 int skew_sync_status(skew_handle_t *h, void *stream) {
     if (!h) return SKEW_EINVAL;

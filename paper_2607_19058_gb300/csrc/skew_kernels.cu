@@ -1,21 +1,31 @@
 // Device kernels of libskewadam (sm_103a).
 //
-// One SkewAdam step (paper Sec. 3, Eq. 1, Algorithm 1) over every tensor of a
-// handle, as four grouped launches over device-side item tables:
-//   k_sumsq    : per-row and per-column sums of g^2 of every factored matrix
-//                (Eq. 1), 16-byte bf16 loads, warp-shuffle row sums, column
-//                partials reduced across the CTA in shared memory and written
-//                per row tile (deterministic: no float atomics);
-//   k_finalize : R <- b2 R + (1-b2) mean_c(G^2), C <- b2 C + (1-b2) mean_r(G^2),
-//                1/sqrt(C_j) per column, and mean(R) by the last item of a tensor;
-//   k_rms      : the tier's momentum / exact second moment update, U up to its
-//                scalar coefficient, and sum(U^2) per tile; the last tile of a
-//                tensor forms RMS(U) and the clip factor (Sec. 3 update clipping);
-//   k_apply    : x = w (1 - lr*lambda) - lr*kappa*U in fp32 and the dithered
-//                bf16 write-back with a Philox-4x32-10 counter hash.
+// One SkewAdam step (paper Sec. 3, Eq. 1, Algorithm 1). The work of a tensor is
+// four phases of tiles / items, each a grouped launch over an item table:
+//   A k_sumsq    : per-row and per-column sums of g^2 of a factored matrix
+//                  (Eq. 1): 16-byte bf16 loads issued eight rows at a time,
+//                  warp-shuffle row sums, column partials reduced across the CTA
+//                  in shared memory and written per row tile (no float atomics);
+//   F k_finalize : R <- b2 R + (1-b2) mean_c(G^2), C <- b2 C + (1-b2) mean_r(G^2),
+//                  1/sqrt(C_j) per column; the last item of a tensor forms mean(R);
+//   B k_rms      : the tier's momentum / exact second-moment update, U up to its
+//                  scalar coefficient and a compensated sum(U^2) per tile; the
+//                  last tile of a tensor forms RMS(U) and the clip factor
+//                  (Sec. 3 update clipping);
+//   C k_apply    : x = w (1 - lr*lambda) - lr*kappa*U in fp32 and the dithered
+//                  bf16 write-back with a Philox-4x32-10 counter hash.
 // The reconstructed second moment of a factored matrix is never formed:
 // 1/sqrt(max(R_i C_j / Rbar, eps)) = min(a_i * b_j, 1/sqrt(eps)) with
-// a_i = 1/sqrt(R_i / Rbar) per row and b_j = 1/sqrt(C_j) per column.
+// a_i = 1/sqrt(R_i / Rbar) per row and b_j = 1/sqrt(C_j) per column, both
+// computed once per tile into shared memory.
+//
+// The host runs a step as one CUDA graph in which each unit of tensors is a
+// chain A -> F -> B -> C on one of several streams; a unit's gradient is loaded
+// from HBM in phase A with an L2 evict-last policy and is still in the L2 when
+// B and C re-read it, while weights stream through with an evict-first policy.
+// The per-step scalars come from a device parameter block (StepArgs), so the
+// graph is launched unchanged every step. Values produced by an earlier phase
+// of the same step are read with L2-only (.cg) loads.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -25,40 +35,80 @@ namespace skew {
 namespace {
 
 constexpr uint32_t kAll = 0xFFFFFFFFu;
+
+// Resident CTAs per SM each kernel is compiled for (register budget 64K / (256 * n)).
+#ifndef SKEW_MINB_SUMSQ
+#define SKEW_MINB_SUMSQ 4
+#endif
+#ifndef SKEW_MINB_RMS
+#define SKEW_MINB_RMS 3
+#endif
+#ifndef SKEW_MINB_APPLY
+#define SKEW_MINB_APPLY 3
+#endif
 constexpr int kSmemFloats = kVecPerThread * kThreads;  // row scales of the tallest tile
+constexpr int kStripCols = 8 * 32;                     // widest column strip
 
 // ---------------------------------------------------------------------------
-// Small helpers
+// Memory access helpers
 // ---------------------------------------------------------------------------
+// L2 eviction policies for 16-byte accesses (created once per thread).
+struct Pol {
+    uint64_t keep;  // evict_last: gradient between its first and last pass
+    uint64_t drop;  // evict_first: streamed once (weights, last gradient read)
+    __device__ Pol() {
+        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(drop));
+    }
+};
+
+__device__ __forceinline__ uint4 ld16_hint(const void *p, uint64_t pol) {
+    uint4 u;
+    asm volatile("ld.global.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
+                 : "=r"(u.x), "=r"(u.y), "=r"(u.z), "=r"(u.w)
+                 : "l"(p), "l"(pol));
+    return u;
+}
+
+__device__ __forceinline__ void st16_hint(void *p, uint4 u, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v4.u32 [%0], {%1,%2,%3,%4}, %5;" ::"l"(p), "r"(u.x), "r"(u.y), "r"(u.z),
+                 "r"(u.w), "l"(pol));
+}
+
 __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float(uint32_t(h) << 16); }
 
-// Eight bf16 values at p (16-byte aligned when VEC) -> fp32; lanes >= valid read as 0.
-template <bool VEC>
-__device__ __forceinline__ void load_bf8(const uint16_t *p, int valid, float (&o)[8]) {
-    if (VEC) {
-        const uint4 u = *reinterpret_cast<const uint4 *>(p);
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+__device__ __forceinline__ void unpack_bf8(uint4 u, float (&o)[8]) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            o[2 * q] = __uint_as_float(w[q] << 16);
-            o[2 * q + 1] = __uint_as_float(w[q] & 0xFFFF0000u);
-        }
-    } else {
-#pragma unroll
-        for (int c = 0; c < 8; ++c) o[c] = c < valid ? bf16_to_f32(p[c]) : 0.f;
+    for (int q = 0; q < 4; ++q) {
+        o[2 * q] = __uint_as_float(w[q] << 16);
+        o[2 * q + 1] = __uint_as_float(w[q] & 0xFFFF0000u);
     }
 }
 
+// Eight bf16 values (scalar path: elements >= valid read as 0).
+__device__ __forceinline__ void load_bf8_scalar(const uint16_t *p, int valid, float (&o)[8]) {
+#pragma unroll
+    for (int c = 0; c < 8; ++c) o[c] = c < valid ? bf16_to_f32(p[c]) : 0.f;
+}
+
+// Eight fp32 values; `cg` reads through L2 only (values an earlier phase wrote).
 template <bool VEC>
-__device__ __forceinline__ void load_f8(const float *p, int valid, float (&o)[8]) {
+__device__ __forceinline__ void load_f8(const float *p, int valid, float (&o)[8], bool cg) {
     if (VEC) {
-        const float4 a = *reinterpret_cast<const float4 *>(p);
-        const float4 b = *reinterpret_cast<const float4 *>(p + 4);
+        float4 a, b;
+        if (cg) {
+            a = __ldcg(reinterpret_cast<const float4 *>(p));
+            b = __ldcg(reinterpret_cast<const float4 *>(p + 4));
+        } else {
+            a = *reinterpret_cast<const float4 *>(p);
+            b = *reinterpret_cast<const float4 *>(p + 4);
+        }
         o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
         o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
     } else {
 #pragma unroll
-        for (int c = 0; c < 8; ++c) o[c] = c < valid ? p[c] : 0.f;
+        for (int c = 0; c < 8; ++c) o[c] = c < valid ? (cg ? __ldcg(p + c) : p[c]) : 0.f;
     }
 }
 
@@ -74,9 +124,11 @@ __device__ __forceinline__ void store_f8(float *p, int valid, const float (&o)[8
     }
 }
 
-// Philox-4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two 32x32
-// multiplies whose high halves are xored with the other counter words and the
-// round key; the key advances by two Weyl constants between rounds.
+// ---------------------------------------------------------------------------
+// Dither: Philox-4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) -- ten rounds of
+// two 32x32 multiplies whose high halves are xored with the other counter
+// words and the round key; the key advances by two Weyl constants per round.
+// ---------------------------------------------------------------------------
 __device__ __forceinline__ uint4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3, uint32_t k0,
                                                uint32_t k1) {
 #pragma unroll
@@ -93,12 +145,20 @@ __device__ __forceinline__ uint4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_
     return make_uint4(c0, c1, c2, c3);
 }
 
+// Dither key of one tensor at one step: tensor id, low 32 bits of the step and
+// the two halves of the seed (kept in registers by the hot loops).
+struct Dith {
+    uint32_t tid, step, k0, k1;
+};
+
+__device__ __forceinline__ Dith dith_of(const StepArgs &A, uint32_t tid) { return Dith{tid, A.step_lo, A.seed_lo, A.seed_hi}; }
+
 // The 16-bit dithers of the eight elements idx0 .. idx0+7 (idx0 a multiple of 8):
 // counter (idx0/8 lo, idx0/8 hi, tensor id, step lo), key (seed lo, seed hi);
 // element k takes half (k & 1) of word k >> 1.
-__device__ __forceinline__ void dither8(uint64_t idx0, uint32_t tid, const StepArgs &A, uint32_t (&r)[8]) {
+__device__ __forceinline__ void dither8(uint64_t idx0, const Dith &d, uint32_t (&r)[8]) {
     const uint64_t blk = idx0 >> 3;
-    const uint4 o = philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), tid, A.step_lo, A.seed_lo, A.seed_hi);
+    const uint4 o = philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), d.tid, d.step, d.k0, d.k1);
     const uint32_t w[4] = {o.x, o.y, o.z, o.w};
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
@@ -107,9 +167,9 @@ __device__ __forceinline__ void dither8(uint64_t idx0, uint32_t tid, const StepA
     }
 }
 
-__device__ __forceinline__ uint32_t dither1(uint64_t idx, uint32_t tid, const StepArgs &A) {
+__device__ __forceinline__ uint32_t dither1(uint64_t idx, const Dith &d) {
     const uint64_t blk = idx >> 3;
-    const uint4 o = philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), tid, A.step_lo, A.seed_lo, A.seed_hi);
+    const uint4 o = philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), d.tid, d.step, d.k0, d.k1);
     const uint32_t k = (uint32_t)(idx & 7);
     const uint32_t w = k < 2 ? o.x : k < 4 ? o.y : k < 6 ? o.z : o.w;
     return (w >> (16 * (k & 1))) & 0xFFFFu;
@@ -129,6 +189,9 @@ __device__ __forceinline__ float row_scale(float Ri, float rbar_s, int rbar_e) {
     return __frsqrt_rn(__fdiv_rn(ldexpf(Ri, rbar_e), rbar_s));
 }
 
+// ---------------------------------------------------------------------------
+// Reductions
+// ---------------------------------------------------------------------------
 // Error-free sum (Knuth's TwoSum): s + e == a + b exactly.
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     s = a + b;
@@ -182,12 +245,6 @@ __device__ float2 block_sum2(Acc2 a, float2 *red) {
     return make_float2(r.hi, r.lo);
 }
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(kAll, v, o);
-    return v;
-}
-
 __device__ __forceinline__ double warp_sum_d(double v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(kAll, v, o);
@@ -209,16 +266,39 @@ __device__ double block_sum_d(double v, double *red) {
     return r;  // valid in thread 0
 }
 
+// Counter increment that publishes this CTA's (barrier-ordered) writes and, for
+// the CTA that sees the final count, acquires every other CTA's.
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t *p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+// Shared scratch of a CTA.
+struct Smem {
+    float colred[kThreads * 8];  // column partials of a sum-of-squares tile
+    float2 red2[kThreads / 32];
+    double redd[kThreads / 32];
+    int last;
+};
+
+// Row scales a_i of a factored tile's rows and column scales b_j of its strip.
+struct Meta {
+    float rows[kSmemFloats];
+    float cols[kStripCols];
+};
+
 // Geometry of a factored tile: LC lanes along a row, RG row groups, 16 rows per thread.
 struct FactTile {
-    uint32_t LC, RG, lane, rg;
+    uint32_t LC, RG, lane, rg, s, rt;
     int64_t col0, row0;
     int valid;
     bool act;
     __device__ FactTile(const TensorDev &T, uint32_t tile) {
         LC = 1u << T.lcl;
         RG = kThreads >> T.lcl;
-        const uint32_t s = tile % T.strips, rt = tile / T.strips;
+        s = tile % T.strips;
+        rt = tile / T.strips;
         lane = threadIdx.x & (LC - 1);
         rg = threadIdx.x >> T.lcl;
         col0 = int64_t(s) * 8 * LC + 8 * lane;
@@ -228,82 +308,154 @@ struct FactTile {
     }
 };
 
+// a_i of the tile's rows and b_j of its strip (R, 1/sqrt(C), mean(R) read from L2).
+__device__ void fill_meta(const TensorDev &T, const TensorScal &S, uint32_t tile, Meta &meta) {
+    const uint32_t s = tile % T.strips, rt = tile / T.strips, width = 8u << T.lcl;
+    const float rbar_s = __ldcg(&S.rbar_s);
+    const int rbar_e = __ldcg(&S.rbar_e);
+    for (uint32_t r = threadIdx.x; r < T.tile_rows; r += kThreads) {
+        const int64_t i = int64_t(rt) * T.tile_rows + r;
+        meta.rows[r] = i < T.n ? row_scale(__ldcg(T.R + i), rbar_s, rbar_e) : 0.f;
+    }
+    for (uint32_t c = threadIdx.x; c < width; c += kThreads) {
+        const int64_t j = int64_t(s) * width + c;
+        meta.cols[c] = j < T.m ? __ldcg(T.bsc + j) : 0.f;
+    }
+    __syncthreads();
+}
+
 // ---------------------------------------------------------------------------
-// Phase 1: per-row / per-column sums of g^2 (Eq. 1).
+// Phase A: per-row / per-column sums of g^2 (Eq. 1).
 // ---------------------------------------------------------------------------
+// Adds the squares of one row-vector to the column partials; returns the row's
+// sum over the LC lanes that share the row.
+__device__ __forceinline__ float sumsq_row(const float (&g)[8], float (&col)[8], uint32_t LC) {
+    float rs = 0.f;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        const float q = g[c] * g[c];
+        col[c] += q;
+        rs += q;
+    }
+    for (uint32_t o = LC >> 1; o; o >>= 1) rs += __shfl_xor_sync(kAll, rs, o);
+    return rs;
+}
+
 template <bool VEC>
-__device__ void sumsq_tile(const TensorDev &T, uint32_t tile, float *sm) {
+__device__ void sumsq_tile(const TensorDev &T, uint32_t tile, Smem &sm, const Pol &pol) {
     const FactTile F(T, tile);
-    const uint32_t s = tile % T.strips, rt = tile / T.strips;
+    const uint16_t *__restrict__ g_ = T.g;
+    float *__restrict__ rowp = T.rowp + int64_t(F.s) * T.n;
+    const int64_t n = T.n, m = T.m, row0 = F.row0, RG = F.RG, col0 = F.col0;
+    const uint32_t LC = F.LC;
+    const bool act = F.act, lane0 = F.lane == 0;
     float col[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
-    for (int k = 0; k < kVecPerThread; ++k) {
-        const int64_t i = F.row0 + int64_t(k) * F.RG;
-        float g[8];
-        if (F.act && i < T.n)
-            load_bf8<VEC>(T.g + i * T.m + F.col0, F.valid, g);
-        else
+    if constexpr (VEC) {
+        constexpr int KCH = 8;  // row-vectors requested before the first is used
+#pragma unroll 1
+        for (int k0 = 0; k0 < kVecPerThread; k0 += KCH) {
+            uint4 raw[KCH];
 #pragma unroll
-            for (int c = 0; c < 8; ++c) g[c] = 0.f;
-        float rs = 0.f;
+            for (int q = 0; q < KCH; ++q) {
+                const int64_t i = row0 + (k0 + q) * RG;
+                raw[q] = (act && i < n) ? ld16_hint(g_ + i * m + col0, pol.keep) : make_uint4(0, 0, 0, 0);
+            }
+            if (LC == 32) {
+                // each lane holds partial sums of 8 rows; a transposed butterfly leaves
+                // lane L with the full sum of row 4*b4 + 2*b3 + b2 (bits of L)
+                float rs[KCH];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-            const float q = g[c] * g[c];
-            col[c] += q;
-            rs += q;
+                for (int q = 0; q < KCH; ++q) {
+                    float g[8];
+                    unpack_bf8(raw[q], g);
+                    float acc = 0.f;
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const float sq = g[c] * g[c];
+                        col[c] += sq;
+                        acc += sq;
+                    }
+                    rs[q] = acc;
+                }
+                const uint32_t ln = threadIdx.x & 31;
+                const bool b4 = ln & 16, b3 = ln & 8, b2 = ln & 4;
+                float v4[4], v2[2];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float keep = b4 ? rs[q + 4] : rs[q], send = b4 ? rs[q] : rs[q + 4];
+                    v4[q] = keep + __shfl_xor_sync(kAll, send, 16);
+                }
+#pragma unroll
+                for (int q = 0; q < 2; ++q) {
+                    const float keep = b3 ? v4[q + 2] : v4[q], send = b3 ? v4[q] : v4[q + 2];
+                    v2[q] = keep + __shfl_xor_sync(kAll, send, 8);
+                }
+                float v1 = (b2 ? v2[1] : v2[0]) + __shfl_xor_sync(kAll, b2 ? v2[0] : v2[1], 4);
+                v1 += __shfl_xor_sync(kAll, v1, 2);
+                v1 += __shfl_xor_sync(kAll, v1, 1);
+                const int qs = (b4 ? 4 : 0) + (b3 ? 2 : 0) + (b2 ? 1 : 0);
+                const int64_t i = row0 + (k0 + qs) * RG;
+                if ((ln & 3) == 0 && i < n) rowp[i] = v1;
+            } else {
+#pragma unroll
+                for (int q = 0; q < KCH; ++q) {
+                    const int64_t i = row0 + (k0 + q) * RG;
+                    float g[8];
+                    unpack_bf8(raw[q], g);
+                    const float rs = sumsq_row(g, col, LC);
+                    if (lane0 && i < n) rowp[i] = rs;
+                }
+            }
         }
-        for (uint32_t o = F.LC >> 1; o; o >>= 1) rs += __shfl_xor_sync(kAll, rs, o);
-        if (F.lane == 0 && i < T.n) T.rowp[int64_t(s) * T.n + i] = rs;
+    } else {
+        for (int k = 0; k < kVecPerThread; ++k) {
+            const int64_t i = row0 + k * RG;
+            float g[8];
+            if (act && i < n)
+                load_bf8_scalar(g_ + i * m + col0, F.valid, g);
+            else
+#pragma unroll
+                for (int c = 0; c < 8; ++c) g[c] = 0.f;
+            const float rs = sumsq_row(g, col, LC);
+            if (lane0 && i < n) rowp[i] = rs;
+        }
     }
 #pragma unroll
-    for (int c = 0; c < 8; ++c) sm[threadIdx.x * 8 + c] = col[c];
+    for (int c = 0; c < 8; ++c) sm.colred[threadIdx.x * 8 + c] = col[c];
     __syncthreads();
-    const uint32_t width = 8 * F.LC;
+    const uint32_t width = 8 * LC;
     for (uint32_t cc = threadIdx.x; cc < width; cc += kThreads) {
         float acc = 0.f;
-        for (uint32_t r = 0; r < F.RG; ++r) acc += sm[r * width + cc];
-        const int64_t j = int64_t(s) * width + cc;
-        if (j < T.m) T.colp[int64_t(rt) * T.m + j] = acc;
+        for (uint32_t r = 0; r < F.RG; ++r) acc += sm.colred[r * width + cc];
+        const int64_t j = int64_t(F.s) * width + cc;
+        if (j < m) T.colp[int64_t(F.rt) * m + j] = acc;
     }
 }
 
-__global__ void __launch_bounds__(kThreads) k_sumsq(StepArgs A) {
-    __shared__ float sm[kThreads * 8];
-    const uint2 it = A.items[blockIdx.x];
-    const TensorDev &T = A.tensors[it.x];
-    if (T.vec)
-        sumsq_tile<true>(T, it.y, sm);
-    else
-        sumsq_tile<false>(T, it.y, sm);
-}
-
 // ---------------------------------------------------------------------------
-// Phase 2: factor EMAs, 1/sqrt(C_j), mean(R) (Eq. 1).
+// Phase F: factor EMAs, 1/sqrt(C_j), mean(R) (Eq. 1).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) k_finalize(StepArgs A) {
-    __shared__ double red[kThreads / 32];
-    __shared__ int last;
-    const uint2 it = A.items[blockIdx.x];
-    const TensorDev &T = A.tensors[it.x];
-    TensorScal &S = A.scal[it.x];
-    if (it.y < T.nfr) {
-        const int64_t i = int64_t(it.y) * kFinChunk + threadIdx.x;
+__device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm) {
+    const TensorDev &T = A.tensors[t];
+    TensorScal &S = A.scal[t];
+    if (local < T.nfr) {
+        const int64_t i = int64_t(local) * kFinChunk + threadIdx.x;
         double rd = 0.0;
-        if (i < T.n) {
+        if (threadIdx.x < kFinChunk && i < T.n) {
             float rs = 0.f;
-            for (uint32_t s = 0; s < T.strips; ++s) rs += T.rowp[int64_t(s) * T.n + i];
+            for (uint32_t s = 0; s < T.strips; ++s) rs += __ldcg(T.rowp + int64_t(s) * T.n + i);
             const float mean = __fdiv_rn(rs, (float)T.m);
             const float Rn = fmaf(A.b2, T.R[i], A.c2 * mean);
             T.R[i] = Rn;
             rd = (double)Rn;
         }
-        rd = block_sum_d(rd, red);
-        if (threadIdx.x == 0) T.rsum[it.y] = rd;
+        rd = block_sum_d(rd, sm.redd);
+        if (threadIdx.x == 0) T.rsum[local] = rd;
     } else {
-        const int64_t j = int64_t(it.y - T.nfr) * kFinChunk + threadIdx.x;
-        if (j < T.m) {
+        const int64_t j = int64_t(local - T.nfr) * kFinChunk + threadIdx.x;
+        if (threadIdx.x < kFinChunk && j < T.m) {
             float cs = 0.f;
-            for (uint32_t r = 0; r < T.rowtiles; ++r) cs += T.colp[int64_t(r) * T.m + j];
+            for (uint32_t r = 0; r < T.rowtiles; ++r) cs += __ldcg(T.colp + int64_t(r) * T.m + j);
             const float mean = __fdiv_rn(cs, (float)T.n);
             const float Cn = fmaf(A.b2, T.C[j], A.c2 * mean);
             T.C[j] = Cn;
@@ -312,14 +464,9 @@ __global__ void __launch_bounds__(kThreads) k_finalize(StepArgs A) {
     }
     // The last finalize item of the tensor forms mean(R) from the row items' partial sums.
     __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        const uint32_t done = atomicAdd(&S.cntF, 1u);
-        last = (done == T.nfr + T.nfc - 1);
-    }
+    if (threadIdx.x == 0) sm.last = (atom_add_acq_rel(&S.cntF, 1u) == T.nfr + T.nfc - 1);
     __syncthreads();
-    if (last && threadIdx.x == 0) {
-        __threadfence();
+    if (sm.last && threadIdx.x == 0) {
         double s = 0.0;
         for (uint32_t f = 0; f < T.nfr; ++f) s += __ldcg(T.rsum + f);
         const double rbar = s / (double)T.n;
@@ -337,61 +484,104 @@ __global__ void __launch_bounds__(kThreads) k_finalize(StepArgs A) {
 }
 
 // ---------------------------------------------------------------------------
-// Phase 3: second moment / momentum update and sum(U^2) (Algorithm 1).
+// Phase B: second moment / momentum update and sum(U^2) (Algorithm 1).
 // ---------------------------------------------------------------------------
-template <bool VEC>
-__device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile, float *sm) {
+// U (up to its scalar) of one row-vector of a factored tile, squared and summed into acc.
+__device__ __forceinline__ void rms_row(const float (&y)[8], float a, const float (&b)[8], int valid, float ce,
+                                        Acc2 &acc) {
+    float u[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) u[c] = c < valid ? y[c] * fminf(a * b[c], ce) : 0.f;
+    acc.add(sumsq8(u));
+}
+
+template <bool VEC, bool MOM>
+__device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t tile, const Meta &meta,
+                              const Pol &pol) {
     const FactTile F(T, tile);
-    const uint32_t rt = tile / T.strips;
-    for (uint32_t r = threadIdx.x; r < T.tile_rows; r += kThreads) {
-        const int64_t i = int64_t(rt) * T.tile_rows + r;
-        sm[r] = i < T.n ? row_scale(T.R[i], S.rbar_s, S.rbar_e) : 0.f;
-    }
-    __syncthreads();
-    float b[8];
-    if (F.act)
-        load_f8<VEC>(T.bsc + F.col0, F.valid, b);
     Acc2 acc;
     if (!F.act) return acc;
-#pragma unroll 2
-    for (int k = 0; k < kVecPerThread; ++k) {
-        const int64_t i = F.row0 + int64_t(k) * F.RG;
-        if (i >= T.n) break;
-        const int64_t e0 = i * T.m + F.col0;
-        float y[8];
-        load_bf8<VEC>(T.g + e0, F.valid, y);
-        if (T.momentum) {
-            float mm[8];
-            load_f8<VEC>(T.M + e0, F.valid, mm);
+    const uint16_t *__restrict__ g_ = T.g;
+    float *__restrict__ M_ = T.M;
+    const int64_t n = T.n, m = T.m, row0 = F.row0, RG = F.RG, col0 = F.col0;
+    const int valid = F.valid;
+    const float b1 = A.b1, c1 = A.c1, ce = A.ce;
+    const float *rows = meta.rows + F.rg;
+    float b[8];
 #pragma unroll
-            for (int c = 0; c < 8; ++c) y[c] = fmaf(A.b1, mm[c], A.c1 * y[c]);
-            store_f8<VEC>(T.M + e0, F.valid, y);
+    for (int c = 0; c < 8; ++c) b[c] = meta.cols[F.lane * 8 + c];
+    if constexpr (VEC) {
+        // row-vectors requested together: eight when only g streams, four with the momentum
+        constexpr int KCH = MOM ? 4 : 8;
+#pragma unroll 1
+        for (int k0 = 0; k0 < kVecPerThread; k0 += KCH) {
+            uint4 graw[KCH];
+            float4 mraw[MOM ? KCH : 1][2];
+#pragma unroll
+            for (int q = 0; q < KCH; ++q) {
+                const int64_t i = row0 + (k0 + q) * RG;
+                const int64_t e0 = (i < n ? i : 0) * m + col0;
+                if (i < n) graw[q] = ld16_hint(g_ + e0, MOM ? pol.drop : pol.keep);
+                if (MOM && i < n) {
+                    mraw[MOM ? q : 0][0] = *reinterpret_cast<const float4 *>(M_ + e0);
+                    mraw[MOM ? q : 0][1] = *reinterpret_cast<const float4 *>(M_ + e0 + 4);
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < KCH; ++q) {
+                const int64_t i = row0 + (k0 + q) * RG;
+                if (i < n) {
+                    float y[8];
+                    unpack_bf8(graw[q], y);
+                    if (MOM) {
+                        const float4 m0 = mraw[MOM ? q : 0][0], m1 = mraw[MOM ? q : 0][1];
+                        const float mm[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) y[c] = fmaf(b1, mm[c], c1 * y[c]);
+                        store_f8<true>(M_ + i * m + col0, 8, y);
+                    }
+                    rms_row(y, rows[(k0 + q) * RG], b, 8, ce, acc);
+                }
+            }
         }
-        const float a = sm[F.rg + k * F.RG];
-        float u[8];
+    } else {
+        for (int k = 0; k < kVecPerThread; ++k) {
+            const int64_t i = row0 + k * RG;
+            if (i >= n) break;
+            float y[8];
+            load_bf8_scalar(g_ + i * m + col0, valid, y);
+            if (MOM) {
+                float mm[8];
+                load_f8<false>(M_ + i * m + col0, valid, mm, false);
 #pragma unroll
-        for (int c = 0; c < 8; ++c) u[c] = c < F.valid ? y[c] * fminf(a * b[c], A.ce) : 0.f;
-        acc.add(sumsq8(u));
+                for (int c = 0; c < 8; ++c) y[c] = fmaf(b1, mm[c], c1 * y[c]);
+                store_f8<false>(M_ + i * m + col0, valid, y);
+            }
+            rms_row(y, rows[k * RG], b, valid, ce, acc);
+        }
     }
     return acc;
 }
 
 template <bool VEC>
-__device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t tile) {
+__device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t tile, const Pol &pol) {
     Acc2 acc;
     for (int k = 0; k < kVecPerThread; ++k) {
         const int64_t e0 = 8 * (int64_t(tile) * kThreads * kVecPerThread + int64_t(k) * kThreads + threadIdx.x);
         if (e0 >= T.numel) break;
         const int valid = (int)min(int64_t(8), T.numel - e0);
         float g[8], v[8], y[8];
-        load_bf8<VEC>(T.g + e0, valid, g);
-        load_f8<VEC>(T.v + e0, valid, v);
+        if (VEC)
+            unpack_bf8(ld16_hint(T.g + e0, pol.drop), g);
+        else
+            load_bf8_scalar(T.g + e0, valid, g);
+        load_f8<VEC>(T.v + e0, valid, v, false);
 #pragma unroll
         for (int c = 0; c < 8; ++c) v[c] = fmaf(A.b2, v[c], A.c2 * (g[c] * g[c]));
         store_f8<VEC>(T.v + e0, valid, v);
         if (T.momentum) {
             float mm[8];
-            load_f8<VEC>(T.M + e0, valid, mm);
+            load_f8<VEC>(T.M + e0, valid, mm, false);
 #pragma unroll
             for (int c = 0; c < 8; ++c) y[c] = fmaf(A.b1, mm[c], A.c1 * g[c]);
             store_f8<VEC>(T.M + e0, valid, y);
@@ -407,36 +597,34 @@ __device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
     return acc;
 }
 
-__global__ void __launch_bounds__(kThreads) k_rms(StepArgs A) {
-    __shared__ float sm[kSmemFloats];
-    __shared__ float2 red[kThreads / 32];
-    __shared__ double redd[kThreads / 32];
-    __shared__ int last;
-    const uint2 it = A.items[blockIdx.x];
-    const TensorDev &T = A.tensors[it.x];
-    TensorScal &S = A.scal[it.x];
+__device__ void phase_B(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm, const Meta &meta, const Pol &pol) {
+    const TensorDev &T = A.tensors[t];
+    TensorScal &S = A.scal[t];
     Acc2 acc;
-    if (T.kind == kKindFactored)
-        acc = T.vec ? rms_fact_tile<true>(A, T, S, it.y, sm) : rms_fact_tile<false>(A, T, S, it.y, sm);
-    else
-        acc = T.vec ? rms_full_tile<true>(A, T, it.y) : rms_full_tile<false>(A, T, it.y);
-    const float2 tsum = block_sum2(acc, red);
+    if (T.kind == kKindFactored) {
+        if (T.vec)
+            acc = T.momentum ? rms_fact_tile<true, true>(A, T, local, meta, pol)
+                             : rms_fact_tile<true, false>(A, T, local, meta, pol);
+        else
+            acc = T.momentum ? rms_fact_tile<false, true>(A, T, local, meta, pol)
+                             : rms_fact_tile<false, false>(A, T, local, meta, pol);
+    } else {
+        acc = T.vec ? rms_full_tile<true>(A, T, local, pol) : rms_full_tile<false>(A, T, local, pol);
+    }
+    const float2 tsum = block_sum2(acc, sm.red2);
     if (threadIdx.x == 0) {
-        T.u2[it.y] = tsum;
-        __threadfence();
-        const uint32_t done = atomicAdd(&S.cntB, 1u);
-        last = (done == T.ntiles - 1);
+        T.u2[local] = tsum;
+        sm.last = (atom_add_acq_rel(&S.cntB, 1u) == T.ntiles - 1);
     }
     __syncthreads();
-    if (!last) return;
+    if (!sm.last) return;
     // Last tile of the tensor: sum(U^2), RMS, clip factor (fixed summation order).
-    __threadfence();
     double s = 0.0;
     for (uint32_t k = threadIdx.x; k < T.ntiles; k += kThreads) {
         const float2 p = __ldcg(T.u2 + k);
         s += (double)p.x + (double)p.y;
     }
-    s = block_sum_d(s, redd);
+    s = block_sum_d(s, sm.redd);
     if (threadIdx.x == 0) {
         const double coef = T.momentum ? A.coef_mom : A.coef_plain;
         const double su2 = s * coef * coef;
@@ -450,66 +638,122 @@ __global__ void __launch_bounds__(kThreads) k_rms(StepArgs A) {
 }
 
 // ---------------------------------------------------------------------------
-// Phase 4: decoupled decay, clipped update, dithered bf16 write-back.
+// Phase C: decoupled decay, clipped update, dithered bf16 write-back.
 // ---------------------------------------------------------------------------
+// x of eight elements -> dithered bf16, stored at w + e0 (16-byte store when VEC).
 template <bool VEC>
-__device__ __forceinline__ void write8(const StepArgs &A, const TensorDev &T, int64_t e0, int valid, bool aligned8,
-                                       const float (&x)[8]) {
+__device__ __forceinline__ void write8(uint16_t *__restrict__ w, const Dith &d, int64_t e0, int valid, bool aligned8,
+                                       const float (&x)[8], const Pol &pol) {
+    uint32_t r[8];
     if (VEC) {
-        uint32_t r[8];
-        dither8((uint64_t)e0, T.tid, A, r);
+        dither8((uint64_t)e0, d, r);
         uint32_t o[4];
+        // a NaN anywhere makes the sum NaN (so does Inf - Inf): only then test per element
+        const float any = ((x[0] + x[1]) + (x[2] + x[3])) + ((x[4] + x[5]) + (x[6] + x[7]));
+        if (any == any) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) o[q] = sr_bf16(x[2 * q], r[2 * q]) | (sr_bf16(x[2 * q + 1], r[2 * q + 1]) << 16);
-        *reinterpret_cast<uint4 *>(T.w + e0) = make_uint4(o[0], o[1], o[2], o[3]);
+            for (int q = 0; q < 4; ++q)  // top halves of (bits + draw) of the two elements
+                o[q] = __byte_perm(__float_as_uint(x[2 * q]) + r[2 * q], __float_as_uint(x[2 * q + 1]) + r[2 * q + 1],
+                                   0x7632);
+        } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                o[q] = sr_bf16(x[2 * q], r[2 * q]) | (sr_bf16(x[2 * q + 1], r[2 * q + 1]) << 16);
+        }
+        st16_hint(w + e0, make_uint4(o[0], o[1], o[2], o[3]), pol.drop);
     } else {
-        uint32_t r[8];
-        if (aligned8) dither8((uint64_t)e0, T.tid, A, r);
+        if (aligned8) dither8((uint64_t)e0, d, r);
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
             if (c < valid) {
-                const uint32_t rc = aligned8 ? r[c] : dither1((uint64_t)(e0 + c), T.tid, A);
-                T.w[e0 + c] = (uint16_t)sr_bf16(x[c], rc);
+                const uint32_t rc = aligned8 ? r[c] : dither1((uint64_t)(e0 + c), d);
+                w[e0 + c] = (uint16_t)sr_bf16(x[c], rc);
             }
         }
     }
 }
 
-template <bool VEC>
-__device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile, float *sm) {
+template <bool VEC, bool MOM>
+__device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile,
+                                const Meta &meta, const Pol &pol) {
     const FactTile F(T, tile);
-    const uint32_t rt = tile / T.strips;
-    for (uint32_t r = threadIdx.x; r < T.tile_rows; r += kThreads) {
-        const int64_t i = int64_t(rt) * T.tile_rows + r;
-        sm[r] = i < T.n ? row_scale(T.R[i], S.rbar_s, S.rbar_e) : 0.f;
-    }
-    __syncthreads();
     if (!F.act) return;
-    float b[8];
-    load_f8<VEC>(T.bsc + F.col0, F.valid, b);
-    const float coefC = S.coefC;
+    const uint16_t *__restrict__ g_ = T.g;
+    const float *__restrict__ M_ = T.M;
+    uint16_t *__restrict__ w_ = T.w;
+    const int64_t n = T.n, m = T.m, row0 = F.row0, RG = F.RG, col0 = F.col0;
+    const int valid = F.valid;
+    const Dith d = dith_of(A, T.tid);
+    const float coefC = __ldcg(&S.coefC);
     const float wdf = T.decay ? A.wdf : 1.0f;
-#pragma unroll 2
-    for (int k = 0; k < kVecPerThread; ++k) {
-        const int64_t i = F.row0 + int64_t(k) * F.RG;
-        if (i >= T.n) break;
-        const int64_t e0 = i * T.m + F.col0;
-        float y[8], w[8], x[8];
-        if (T.momentum)
-            load_f8<VEC>(T.M + e0, F.valid, y);
-        else
-            load_bf8<VEC>(T.g + e0, F.valid, y);
-        load_bf8<VEC>(T.w + e0, F.valid, w);
-        const float a = sm[F.rg + k * F.RG];
+    const float ce = A.ce;
+    const float *rows = meta.rows + F.rg;
+    float b[8];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], A.ce), w[c] * wdf);
-        write8<VEC>(A, T, e0, F.valid, (e0 & 7) == 0, x);
+    for (int c = 0; c < 8; ++c) b[c] = meta.cols[F.lane * 8 + c];
+    if constexpr (VEC) {
+        constexpr int KCH = 4;  // row-vectors (with their weights) requested together
+#pragma unroll 1
+        for (int k0 = 0; k0 < kVecPerThread; k0 += KCH) {
+            uint4 wraw[KCH], graw[MOM ? 1 : KCH];
+            float4 mraw[MOM ? KCH : 1][2];
+#pragma unroll
+            for (int q = 0; q < KCH; ++q) {
+                const int64_t i = row0 + (k0 + q) * RG;
+                const int64_t e0 = (i < n ? i : 0) * m + col0;
+                if (i < n) {
+                    if (MOM) {
+                        mraw[MOM ? q : 0][0] = __ldcg(reinterpret_cast<const float4 *>(M_ + e0));
+                        mraw[MOM ? q : 0][1] = __ldcg(reinterpret_cast<const float4 *>(M_ + e0 + 4));
+                    } else {
+                        graw[MOM ? 0 : q] = ld16_hint(g_ + e0, pol.drop);
+                    }
+                    wraw[q] = ld16_hint(w_ + e0, pol.drop);
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < KCH; ++q) {
+                const int64_t i = row0 + (k0 + q) * RG;
+                if (i < n) {
+                    float y[8], w[8], x[8];
+                    if (MOM) {
+                        const float4 m0 = mraw[MOM ? q : 0][0], m1 = mraw[MOM ? q : 0][1];
+                        y[0] = m0.x; y[1] = m0.y; y[2] = m0.z; y[3] = m0.w;
+                        y[4] = m1.x; y[5] = m1.y; y[6] = m1.z; y[7] = m1.w;
+                    } else {
+                        unpack_bf8(graw[MOM ? 0 : q], y);
+                    }
+                    unpack_bf8(wraw[q], w);
+                    const float a = rows[(k0 + q) * RG];
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], ce), w[c] * wdf);
+                    write8<true>(w_, d, i * m + col0, 8, true, x, pol);
+                }
+            }
+        }
+    } else {
+        for (int k = 0; k < kVecPerThread; ++k) {
+            const int64_t i = row0 + k * RG;
+            if (i >= n) break;
+            const int64_t e0 = i * m + col0;
+            float y[8], w[8], x[8];
+            if (MOM)
+                load_f8<false>(M_ + e0, valid, y, true);
+            else
+                load_bf8_scalar(g_ + e0, valid, y);
+            load_bf8_scalar(w_ + e0, valid, w);
+            const float a = rows[k * RG];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], ce), w[c] * wdf);
+            write8<false>(w_, d, e0, valid, (e0 & 7) == 0, x, pol);
+        }
     }
 }
 
 template <bool VEC>
-__device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile) {
-    const float coefC = S.coefC;
+__device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile,
+                                const Pol &pol) {
+    const float coefC = __ldcg(&S.coefC);
     const float wdf = T.decay ? A.wdf : 1.0f;
     for (int k = 0; k < kVecPerThread; ++k) {
         const int64_t e0 = 8 * (int64_t(tile) * kThreads * kVecPerThread + int64_t(k) * kThreads + threadIdx.x);
@@ -517,63 +761,93 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
         const int valid = (int)min(int64_t(8), T.numel - e0);
         float y[8], v[8], w[8], x[8];
         if (T.momentum)
-            load_f8<VEC>(T.M + e0, valid, y);
+            load_f8<VEC>(T.M + e0, valid, y, true);
+        else if (VEC)
+            unpack_bf8(ld16_hint(T.g + e0, pol.drop), y);
         else
-            load_bf8<VEC>(T.g + e0, valid, y);
-        load_f8<VEC>(T.v + e0, valid, v);
-        load_bf8<VEC>(T.w + e0, valid, w);
+            load_bf8_scalar(T.g + e0, valid, y);
+        load_f8<VEC>(T.v + e0, valid, v, true);
+        if (VEC)
+            unpack_bf8(ld16_hint(T.w + e0, pol.drop), w);
+        else
+            load_bf8_scalar(T.w + e0, valid, w);
 #pragma unroll
         for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(__frsqrt_rn(v[c]), A.ce), w[c] * wdf);
-        write8<VEC>(A, T, e0, valid, true, x);
+        write8<VEC>(T.w, dith_of(A, T.tid), e0, valid, true, x, pol);
     }
 }
 
-__global__ void __launch_bounds__(kThreads) k_apply(StepArgs A) {
-    __shared__ float sm[kSmemFloats];
-    const uint2 it = A.items[blockIdx.x];
+// ---------------------------------------------------------------------------
+// Kernels: one tile / item per CTA, parameters from the device block P.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, SKEW_MINB_SUMSQ) k_sumsq(const StepArgs *__restrict__ P, const uint2 *items) {
+    __shared__ Smem sm;
+    const StepArgs &A = *P;
+    const Pol pol;
+    const uint2 it = items[blockIdx.x];
+    const TensorDev &T = A.tensors[it.x];
+    if (T.vec)
+        sumsq_tile<true>(T, it.y, sm, pol);
+    else
+        sumsq_tile<false>(T, it.y, sm, pol);
+}
+
+__global__ void __launch_bounds__(kThreads) k_finalize(const StepArgs *__restrict__ P, const uint2 *items) {
+    __shared__ Smem sm;
+    const StepArgs &A = *P;
+    const uint2 it = items[blockIdx.x];
+    phase_F(A, it.x, it.y, sm);
+}
+
+__global__ void __launch_bounds__(kThreads, SKEW_MINB_RMS) k_rms(const StepArgs *__restrict__ P, const uint2 *items) {
+    __shared__ Smem sm;
+    __shared__ Meta meta;
+    const StepArgs &A = *P;
+    const Pol pol;
+    const uint2 it = items[blockIdx.x];
+    const TensorDev &T = A.tensors[it.x];
+    if (T.kind == kKindFactored) fill_meta(T, A.scal[it.x], it.y, meta);
+    phase_B(A, it.x, it.y, sm, meta, pol);
+}
+
+__global__ void __launch_bounds__(kThreads, SKEW_MINB_APPLY) k_apply(const StepArgs *__restrict__ P, const uint2 *items) {
+    __shared__ Meta meta;
+    const StepArgs &A = *P;
+    const Pol pol;
+    const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
     const TensorScal &S = A.scal[it.x];
     if (T.kind == kKindFactored) {
-        if (T.vec)
-            apply_fact_tile<true>(A, T, S, it.y, sm);
-        else
-            apply_fact_tile<false>(A, T, S, it.y, sm);
+        fill_meta(T, S, it.y, meta);
+        if (T.vec) {
+            if (T.momentum)
+                apply_fact_tile<true, true>(A, T, S, it.y, meta, pol);
+            else
+                apply_fact_tile<true, false>(A, T, S, it.y, meta, pol);
+        } else {
+            if (T.momentum)
+                apply_fact_tile<false, true>(A, T, S, it.y, meta, pol);
+            else
+                apply_fact_tile<false, false>(A, T, S, it.y, meta, pol);
+        }
     } else {
         if (T.vec)
-            apply_full_tile<true>(A, T, S, it.y);
+            apply_full_tile<true>(A, T, S, it.y, pol);
         else
-            apply_full_tile<false>(A, T, S, it.y);
+            apply_full_tile<false>(A, T, S, it.y, pol);
     }
 }
 
 }  // namespace
 
-const char *const kKernelNames[kNumKernels] = {"k_sumsq", "k_finalize", "k_rms", "k_apply"};
-
-int launch_step(const LaunchPlan &P, const StepArgs &A0, void *stream) {
+int launch_phases(const StepArgs *P, const LaunchPlan &L, void *stream) {
     cudaStream_t s = (cudaStream_t)stream;
-    StepArgs A = A0;
-    auto mark = [&](int k) {
-        if (P.events) cudaEventRecord((cudaEvent_t)P.events[k], s);
-    };
-    mark(0);
-    if (P.nA) {
-        A.items = P.itemsA;
-        k_sumsq<<<P.nA, kThreads, 0, s>>>(A);
+    if (L.nA) k_sumsq<<<L.nA, kThreads, 0, s>>>(P, L.itemsA);
+    if (L.nF) k_finalize<<<L.nF, kThreads, 0, s>>>(P, L.itemsF);
+    if (L.nBC) {
+        k_rms<<<L.nBC, kThreads, 0, s>>>(P, L.itemsBC);
+        k_apply<<<L.nBC, kThreads, 0, s>>>(P, L.itemsBC);
     }
-    mark(1);
-    if (P.nF) {
-        A.items = P.itemsF;
-        k_finalize<<<P.nF, kThreads, 0, s>>>(A);
-    }
-    mark(2);
-    if (P.nBC) {
-        A.items = P.itemsBC;
-        k_rms<<<P.nBC, kThreads, 0, s>>>(A);
-    }
-    mark(3);
-    if (P.nBC) k_apply<<<P.nBC, kThreads, 0, s>>>(A);
-    mark(4);
     return (int)cudaGetLastError();
 }
 

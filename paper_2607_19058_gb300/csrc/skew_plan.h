@@ -11,7 +11,7 @@ namespace skew {
 // (one 16-byte vector) of up to kVecPerThread rows (factored tiles) or flat
 // vectors (full-second-moment tiles). A tile is therefore 32 Ki elements.
 constexpr int kThreads = 256;
-constexpr int kVecPerThread = 16;
+constexpr int kVecPerThread = 32;
 constexpr int64_t kFlatTileElems = int64_t(kThreads) * kVecPerThread * 8;
 constexpr int kFinChunk = 256;  // rows / columns per finalize item
 
@@ -45,7 +45,7 @@ struct TensorDev {
 // Per-tensor scalars of the current step (zeroed at the start of every step).
 struct TensorScal {
     double rbar;      // mean(R)
-    double sumsq;     // sum over the tensor of (U / coef)^2
+    double sumsq;     // sum over the tensor of U^2
     double rms;       // RMS(U)
     double kappa;     // 1 / max(1, RMS / d)
     float rbar_s;     // mean(R) * 2^rbar_e, in [1, 2); 0 if mean(R) == 0
@@ -57,12 +57,11 @@ struct TensorScal {
 };
 static_assert(sizeof(TensorScal) == 64, "TensorScal layout");
 
-// Per-step scalars passed by value to every kernel.
+// Per-step parameters. skew_step writes them into a device-resident block that
+// every kernel reads, so that a captured graph of the step never changes.
 struct StepArgs {
     const TensorDev *tensors;
     TensorScal *scal;
-    const uint2 *items;  // (tensor, local tile / item) for this launch
-    uint32_t *err;
     float b1, b2, c1, c2;  // beta1, beta2, 1-beta1, 1-beta2 (fp32)
     float ce;              // 1 / sqrt(eps), fp32
     float wdf;             // 1 - lr * lambda, fp32
@@ -74,18 +73,15 @@ struct StepArgs {
     uint32_t seed_lo, seed_hi;
 };
 
-// Kernels of one step, in launch order (for per-kernel timing).
-constexpr int kNumKernels = 4;
-extern const char *const kKernelNames[kNumKernels];
-
-// Launch plan of one step (host side).
+// The four phases of a set of tensors: item lists (tensor, local tile / item)
+// in device memory and their lengths.
 struct LaunchPlan {
-    uint32_t nA, nF, nBC;            // items in each phase
+    uint32_t nA, nF, nBC;
     const uint2 *itemsA, *itemsF, *itemsBC;
-    void *const *events;             // null, or kNumKernels + 1 cudaEvent_t recorded around the kernels
 };
 
-// Enqueues the phases of one step; returns a cudaError_t value.
-int launch_step(const LaunchPlan &plan, const StepArgs &args, void *stream);
+// Enqueues the phases of `L` as four grouped launches (A, F, B, C) on `stream`,
+// all reading the parameter block P (device memory); returns a cudaError_t value.
+int launch_phases(const StepArgs *P, const LaunchPlan &L, void *stream);
 
 }  // namespace skew

@@ -27,7 +27,8 @@ KIND_FULL, KIND_FACTORED = 0, 1
 
 EXPORTS = ["skew_create", "skew_destroy", "skew_state_bytes", "skew_workspace_bytes", "skew_bind", "skew_step",
            "skew_sync_status", "skew_tensor_scalars", "skew_tensor_info", "skew_num_tensors", "skew_last_error",
-           "skew_profile_begin", "skew_profile_end", "skew_kernel_name", "skew_step_tensor_noalloc"]
+           "skew_profile_begin", "skew_profile_end", "skew_kernel_name", "skew_step_tensor_noalloc",
+           "skew_launches_per_step"]
 
 
 class SkewError(RuntimeError):
@@ -86,6 +87,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
         L.skew_tensor_scalars.restype = C.c_int
         L.skew_tensor_info.argtypes = [vp, i32, C.POINTER(TensorInfo)]
         L.skew_tensor_info.restype = C.c_int
+        L.skew_launches_per_step.argtypes = [vp]
+        L.skew_launches_per_step.restype = i64
         L.skew_num_tensors.argtypes = [vp]
         L.skew_num_tensors.restype = i32
         L.skew_last_error.argtypes = [vp]
@@ -154,6 +157,10 @@ def skew_tensor_info(h, tid: int) -> TensorInfo:
     info = TensorInfo()
     _check(load().skew_tensor_info(h, tid, C.byref(info)), h)
     return info
+
+
+def skew_launches_per_step(h) -> int:
+    return int(load().skew_launches_per_step(h))
 
 
 def skew_num_tensors(h) -> int:
