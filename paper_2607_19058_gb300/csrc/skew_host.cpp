@@ -36,23 +36,6 @@ thread_local std::string g_create_err;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Integer tuning override from the environment (benchmarking knobs), else `dflt`.
-long env_long(const char *name, long dflt, long lo, long hi) {
-    const char *v = std::getenv(name);
-    if (!v || !*v) return dflt;
-    char *end = nullptr;
-    const long x = std::strtol(v, &end, 10);
-    return (end && *end == 0 && x >= lo && x <= hi) ? x : dflt;
-}
-
-// A unit is a run of consecutive tensors whose phases form one chain of the
-// step graph; its items are ranges of the per-phase item tables.
-struct Unit {
-    uint32_t a0, nA, f0, nF, b0, nBC;
-};
-
-constexpr int kMaxBranches = 8;
-
 }  // namespace
 
 struct skew_handle {
@@ -60,42 +43,23 @@ struct skew_handle {
     skew_hparams_t hp{};
     std::vector<TPlan> t;
     size_t state_bytes = 0, ws_bytes = 0;
-    size_t ws_scal = 0, ws_err = 0, ws_params = 0, ws_tab = 0, ws_tab_end = 0;
+    size_t ws_scal = 0, ws_err = 0, ws_tab = 0, ws_tab_end = 0;
     size_t ws_tens = 0, ws_itemsA = 0, ws_itemsF = 0, ws_itemsBC = 0;
-    std::vector<uint2> itemsA, itemsF, itemsBC;  // unit by unit, tensors in order
-    std::vector<Unit> units;
-    int branches = 3;
+    std::vector<uint2> itemsA, itemsF, itemsBC;  // per phase, tensors in order
     char *state = nullptr, *ws = nullptr;
     bool bound = false;
     std::string err;
-    // the captured step: units round-robin over `branches` streams
-    cudaStream_t br[kMaxBranches] = {};
-    cudaEvent_t fork = nullptr, join[kMaxBranches] = {};
-    cudaGraph_t graph = nullptr;
-    cudaGraphExec_t exec = nullptr;
     // per-launch timing (skew_profile_begin / skew_profile_end)
     std::vector<cudaEvent_t> prof_ev;
     int32_t prof_max = 0, prof_used = 0;
-    void release_graph() {
-        if (exec) cudaGraphExecDestroy(exec);
-        if (graph) cudaGraphDestroy(graph);
-        exec = nullptr;
-        graph = nullptr;
-    }
     ~skew_handle() {
-        release_graph();
-        for (cudaStream_t x : br)
-            if (x) cudaStreamDestroy(x);
-        if (fork) cudaEventDestroy(fork);
-        for (cudaEvent_t e : join)
-            if (e) cudaEventDestroy(e);
         for (cudaEvent_t e : prof_ev) cudaEventDestroy(e);
     }
 };
 
-// What the profiler times per step: the one graph launch.
-constexpr int kProfLaunches = 1;
-const char *const kProfNames[kProfLaunches] = {"step_graph"};
+// What the profiler times per step: the four grouped launches.
+constexpr int kProfLaunches = 4;
+const char *const kProfNames[kProfLaunches] = {"k_sumsq", "k_finalize", "k_rms", "k_apply"};
 
 static int fail(skew_handle_t *h, int code, const char *fmt, ...) {
     char buf[512];
@@ -220,32 +184,16 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
         if (p.kind == kKindFactored) { p.coff = off; off += p.m; }
     h->state_bytes = size_t(off) * 4;
 
-    // Units: consecutive tensors with at least `min_tiles` update tiles (the last
-    // may have fewer), so that one expert matrix is a unit and small tensors are
-    // grouped. Each unit's phases are one chain A -> F -> B -> C of the step graph.
+    // Item tables: every factored tensor's tiles (phase A), finalize items
+    // (phase F) and every tensor's tiles (phases B and C), tensors in order.
     try {
-        const long min_tiles = env_long("SKEW_UNIT_MIN_TILES", 1L << 30, 1, 1L << 30);
-        h->branches = (int)env_long("SKEW_BRANCHES", 1, 1, kMaxBranches);
-        int b = 0;
-        long acc = 0;
-        for (int k = 0; k < n_params; ++k) {
-            acc += h->t[k].ntiles;
-            if (acc < min_tiles && k != n_params - 1) continue;
-            Unit u{(uint32_t)h->itemsA.size(), 0, (uint32_t)h->itemsF.size(), 0, (uint32_t)h->itemsBC.size(), 0};
-            for (int q = b; q <= k; ++q) {
-                const TPlan &p = h->t[q];
-                if (p.kind == kKindFactored) {
-                    for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(q, i));
-                    for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(q, i));
-                }
-                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsBC.push_back(make_uint2(q, i));
+        for (int q = 0; q < n_params; ++q) {
+            const TPlan &p = h->t[q];
+            if (p.kind == kKindFactored) {
+                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(q, i));
+                for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(q, i));
             }
-            u.nA = (uint32_t)h->itemsA.size() - u.a0;
-            u.nF = (uint32_t)h->itemsF.size() - u.f0;
-            u.nBC = (uint32_t)h->itemsBC.size() - u.b0;
-            h->units.push_back(u);
-            b = k + 1;
-            acc = 0;
+            for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsBC.push_back(make_uint2(q, i));
         }
     } catch (...) {
         delete h;
@@ -258,8 +206,6 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     w = align_up(w + sizeof(TensorScal) * n_params, 256);
     h->ws_err = w;
     w = align_up(w + 16, 256);
-    h->ws_params = w;
-    w = align_up(w + sizeof(StepArgs), 256);
     h->ws_tab = w;
     h->ws_tens = w;
     w = align_up(w + sizeof(TensorDev) * n_params, 256);
@@ -298,9 +244,7 @@ int32_t skew_num_tensors(const skew_handle_t *h) { return h ? (int32_t)h->t.size
 
 int64_t skew_launches_per_step(const skew_handle_t *h) {
     if (!h) return 0;
-    int64_t n = 0;
-    for (const Unit &u : h->units) n += (u.nA > 0) + (u.nF > 0) + 2 * (u.nBC > 0);
-    return n;
+    return int64_t(!h->itemsA.empty()) + int64_t(!h->itemsF.empty()) + 2 * int64_t(!h->itemsBC.empty());
 }
 
 const char *skew_last_error(const skew_handle_t *h) { return h ? h->err.c_str() : g_create_err.c_str(); }
@@ -407,41 +351,6 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
     e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(h, e, "bind");
 
-    // Capture the step graph: units round-robin over the branch streams, each a
-    // chain A -> F -> B -> C; the branches fork from and join back to branch 0.
-    h->release_graph();
-    if (!h->units.empty()) {
-        for (int b = 0; b < h->branches; ++b) {
-            if (!h->br[b] && (e = cudaStreamCreateWithFlags(&h->br[b], cudaStreamNonBlocking)) != cudaSuccess)
-                return cuda_fail(h, e, "stream create");
-            if (!h->join[b] && (e = cudaEventCreateWithFlags(&h->join[b], cudaEventDisableTiming)) != cudaSuccess)
-                return cuda_fail(h, e, "event create");
-        }
-        if (!h->fork && (e = cudaEventCreateWithFlags(&h->fork, cudaEventDisableTiming)) != cudaSuccess)
-            return cuda_fail(h, e, "event create");
-        const StepArgs *P = reinterpret_cast<const StepArgs *>(h->ws + h->ws_params);
-        const uint2 *iA = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsA);
-        const uint2 *iF = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsF);
-        const uint2 *iBC = reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsBC);
-        e = cudaStreamBeginCapture(h->br[0], cudaStreamCaptureModeThreadLocal);
-        if (e != cudaSuccess) return cuda_fail(h, e, "graph capture");
-        cudaError_t ce = cudaEventRecord(h->fork, h->br[0]);
-        for (int b = 1; b < h->branches && ce == cudaSuccess; ++b) ce = cudaStreamWaitEvent(h->br[b], h->fork, 0);
-        for (size_t u = 0; u < h->units.size() && ce == cudaSuccess; ++u) {
-            const Unit &U = h->units[u];
-            const LaunchPlan L{U.nA, U.nF, U.nBC, iA + U.a0, iF + U.f0, iBC + U.b0};
-            ce = (cudaError_t)launch_phases(P, L, h->br[u % h->branches]);
-        }
-        for (int b = 1; b < h->branches && ce == cudaSuccess; ++b) {
-            ce = cudaEventRecord(h->join[b], h->br[b]);
-            if (ce == cudaSuccess) ce = cudaStreamWaitEvent(h->br[0], h->join[b], 0);
-        }
-        e = cudaStreamEndCapture(h->br[0], &h->graph);
-        if (ce != cudaSuccess) return cuda_fail(h, ce, "graph capture");
-        if (e != cudaSuccess) return cuda_fail(h, e, "graph capture");
-        e = cudaGraphInstantiate(&h->exec, h->graph, 0);
-        if (e != cudaSuccess) return cuda_fail(h, e, "graph instantiate");
-    }
     h->bound = true;
     return SKEW_OK;
 }
@@ -480,16 +389,14 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
         ev = h->prof_ev.data() + size_t(h->prof_used) * (kProfLaunches + 1);
         ++h->prof_used;
     }
-    // The parameter block: the copy from this pageable struct is staged before
-    // cudaMemcpyAsync returns, so the struct may go out of scope.
-    cudaError_t e = cudaMemcpyAsync(h->ws + h->ws_params, &a, sizeof a, cudaMemcpyHostToDevice, s);
-    if (e != cudaSuccess) return cuda_fail(h, e, "parameter upload");
-    e = cudaMemsetAsync(h->ws + h->ws_scal, 0, sizeof(TensorScal) * h->t.size(), s);
+    cudaError_t e = cudaMemsetAsync(h->ws + h->ws_scal, 0, sizeof(TensorScal) * h->t.size(), s);
     if (e != cudaSuccess) return cuda_fail(h, e, "reset of per-step scalars");
-    if (ev) cudaEventRecord(ev[0], s);
-    e = cudaGraphLaunch(h->exec, s);
-    if (e != cudaSuccess) return cuda_fail(h, e, "graph launch");
-    if (ev) cudaEventRecord(ev[1], s);
+    const LaunchPlan L{(uint32_t)h->itemsA.size(), (uint32_t)h->itemsF.size(), (uint32_t)h->itemsBC.size(),
+                       reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsA),
+                       reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsF),
+                       reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsBC)};
+    e = (cudaError_t)launch_phases(a, L, s, reinterpret_cast<void *const *>(ev));
+    if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
     return SKEW_OK;
 }
 

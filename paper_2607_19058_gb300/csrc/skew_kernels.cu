@@ -19,13 +19,11 @@
 // a_i = 1/sqrt(R_i / Rbar) per row and b_j = 1/sqrt(C_j) per column, both
 // computed once per tile into shared memory.
 //
-// The host runs a step as one CUDA graph in which each unit of tensors is a
-// chain A -> F -> B -> C on one of several streams; a unit's gradient is loaded
-// from HBM in phase A with an L2 evict-last policy and is still in the L2 when
-// B and C re-read it, while weights stream through with an evict-first policy.
-// The per-step scalars come from a device parameter block (StepArgs), so the
-// graph is launched unchanged every step. Values produced by an earlier phase
-// of the same step are read with L2-only (.cg) loads.
+// The host launches the four phases over all tensors, each as one grouped
+// launch (phase-major). The per-step scalars are a kernel parameter (StepArgs,
+// constant bank). Values produced by an earlier phase of the same step are read
+// with L2-only (.cg) loads. When no element of a tile can reach the 1/sqrt(eps)
+// clamp (all but degenerate tiles), phase C takes a clamp-free path.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -286,6 +284,7 @@ struct Smem {
 struct Meta {
     float rows[kSmemFloats];
     float cols[kStripCols];
+    float red[2 * kThreads / 32];  // per-warp maxima of the row / column scales
 };
 
 // Geometry of a factored tile: LC lanes along a row, RG row groups, 16 rows per thread.
@@ -308,20 +307,48 @@ struct FactTile {
     }
 };
 
+// A scale for the clamp-free test: NaN counts as +inf, so that a tile holding a
+// NaN scale never takes the clamp-free path.
+__device__ __forceinline__ float nan_to_inf(float v) { return v == v ? v : __int_as_float(0x7F800000); }
+
 // a_i of the tile's rows and b_j of its strip (R, 1/sqrt(C), mean(R) read from L2).
-__device__ void fill_meta(const TensorDev &T, const TensorScal &S, uint32_t tile, Meta &meta) {
+// Returns (the same value in every thread) whether no element of the tile can
+// reach the clamp: max_i a_i * max_j b_j <= 1/sqrt(eps), all scales finite. Then
+// min(a_i * b_j, 1/sqrt(eps)) = a_i * b_j for every element (rounding is monotone).
+__device__ bool fill_meta(const TensorDev &T, const TensorScal &S, uint32_t tile, float ce, Meta &meta) {
     const uint32_t s = tile % T.strips, rt = tile / T.strips, width = 8u << T.lcl;
     const float rbar_s = __ldcg(&S.rbar_s);
     const int rbar_e = __ldcg(&S.rbar_e);
+    float ma = 0.f, mb = 0.f;
     for (uint32_t r = threadIdx.x; r < T.tile_rows; r += kThreads) {
         const int64_t i = int64_t(rt) * T.tile_rows + r;
-        meta.rows[r] = i < T.n ? row_scale(__ldcg(T.R + i), rbar_s, rbar_e) : 0.f;
+        const float a = i < T.n ? row_scale(__ldcg(T.R + i), rbar_s, rbar_e) : 0.f;
+        meta.rows[r] = a;
+        ma = fmaxf(ma, nan_to_inf(a));
     }
     for (uint32_t c = threadIdx.x; c < width; c += kThreads) {
         const int64_t j = int64_t(s) * width + c;
-        meta.cols[c] = j < T.m ? __ldcg(T.bsc + j) : 0.f;
+        const float b = j < T.m ? __ldcg(T.bsc + j) : 0.f;
+        meta.cols[c] = b;
+        mb = fmaxf(mb, nan_to_inf(b));
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        ma = fmaxf(ma, __shfl_xor_sync(kAll, ma, o));
+        mb = fmaxf(mb, __shfl_xor_sync(kAll, mb, o));
+    }
+    if ((threadIdx.x & 31) == 0) {
+        meta.red[threadIdx.x >> 5] = ma;
+        meta.red[kThreads / 32 + (threadIdx.x >> 5)] = mb;
     }
     __syncthreads();
+    ma = mb = 0.f;
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w) {
+        ma = fmaxf(ma, meta.red[w]);
+        mb = fmaxf(mb, meta.red[kThreads / 32 + w]);
+    }
+    return ma * mb <= ce;
 }
 
 // ---------------------------------------------------------------------------
@@ -673,7 +700,9 @@ __device__ __forceinline__ void write8(uint16_t *__restrict__ w, const Dith &d, 
     }
 }
 
-template <bool VEC, bool MOM>
+// FAST: no element of the tile reaches the clamp (fill_meta), so the update is
+// (-lr*kappa*coef * a_i) * b_j * y, one multiply and one fma per element.
+template <bool VEC, bool MOM, bool FAST>
 __device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile,
                                 const Meta &meta, const Pol &pol) {
     const FactTile F(T, tile);
@@ -725,8 +754,14 @@ __device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const Ten
                     }
                     unpack_bf8(wraw[q], w);
                     const float a = rows[(k0 + q) * RG];
+                    if constexpr (FAST) {
+                        const float ca = -coefC * a;
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], ce), w[c] * wdf);
+                        for (int c = 0; c < 8; ++c) x[c] = fmaf(ca * b[c], y[c], w[c] * wdf);
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], ce), w[c] * wdf);
+                    }
                     write8<true>(w_, d, i * m + col0, 8, true, x, pol);
                 }
             }
@@ -778,11 +813,13 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
 }
 
 // ---------------------------------------------------------------------------
-// Kernels: one tile / item per CTA, parameters from the device block P.
+// Kernels: one tile / item per CTA. The per-step parameters are a kernel
+// parameter (constant bank), so the dither keys and step scalars are uniform
+// operands of every warp.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, SKEW_MINB_SUMSQ) k_sumsq(const StepArgs *__restrict__ P, const uint2 *items) {
+__global__ void __launch_bounds__(kThreads, SKEW_MINB_SUMSQ)
+    k_sumsq(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
     __shared__ Smem sm;
-    const StepArgs &A = *P;
     const Pol pol;
     const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
@@ -792,43 +829,49 @@ __global__ void __launch_bounds__(kThreads, SKEW_MINB_SUMSQ) k_sumsq(const StepA
         sumsq_tile<false>(T, it.y, sm, pol);
 }
 
-__global__ void __launch_bounds__(kThreads) k_finalize(const StepArgs *__restrict__ P, const uint2 *items) {
+__global__ void __launch_bounds__(kThreads) k_finalize(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
     __shared__ Smem sm;
-    const StepArgs &A = *P;
     const uint2 it = items[blockIdx.x];
     phase_F(A, it.x, it.y, sm);
 }
 
-__global__ void __launch_bounds__(kThreads, SKEW_MINB_RMS) k_rms(const StepArgs *__restrict__ P, const uint2 *items) {
+__global__ void __launch_bounds__(kThreads, SKEW_MINB_RMS)
+    k_rms(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
     __shared__ Smem sm;
     __shared__ Meta meta;
-    const StepArgs &A = *P;
     const Pol pol;
     const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
-    if (T.kind == kKindFactored) fill_meta(T, A.scal[it.x], it.y, meta);
+    if (T.kind == kKindFactored) (void)fill_meta(T, A.scal[it.x], it.y, A.ce, meta);
     phase_B(A, it.x, it.y, sm, meta, pol);
 }
 
-__global__ void __launch_bounds__(kThreads, SKEW_MINB_APPLY) k_apply(const StepArgs *__restrict__ P, const uint2 *items) {
+__global__ void __launch_bounds__(kThreads, SKEW_MINB_APPLY)
+    k_apply(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
     __shared__ Meta meta;
-    const StepArgs &A = *P;
     const Pol pol;
     const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
     const TensorScal &S = A.scal[it.x];
     if (T.kind == kKindFactored) {
-        fill_meta(T, S, it.y, meta);
+        const bool fast = fill_meta(T, S, it.y, A.ce, meta);
         if (T.vec) {
-            if (T.momentum)
-                apply_fact_tile<true, true>(A, T, S, it.y, meta, pol);
-            else
-                apply_fact_tile<true, false>(A, T, S, it.y, meta, pol);
+            if (T.momentum) {
+                if (fast)
+                    apply_fact_tile<true, true, true>(A, T, S, it.y, meta, pol);
+                else
+                    apply_fact_tile<true, true, false>(A, T, S, it.y, meta, pol);
+            } else {
+                if (fast)
+                    apply_fact_tile<true, false, true>(A, T, S, it.y, meta, pol);
+                else
+                    apply_fact_tile<true, false, false>(A, T, S, it.y, meta, pol);
+            }
         } else {
             if (T.momentum)
-                apply_fact_tile<false, true>(A, T, S, it.y, meta, pol);
+                apply_fact_tile<false, true, false>(A, T, S, it.y, meta, pol);
             else
-                apply_fact_tile<false, false>(A, T, S, it.y, meta, pol);
+                apply_fact_tile<false, false, false>(A, T, S, it.y, meta, pol);
         }
     } else {
         if (T.vec)
@@ -840,14 +883,20 @@ __global__ void __launch_bounds__(kThreads, SKEW_MINB_APPLY) k_apply(const StepA
 
 }  // namespace
 
-int launch_phases(const StepArgs *P, const LaunchPlan &L, void *stream) {
+int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *const *ev) {
     cudaStream_t s = (cudaStream_t)stream;
-    if (L.nA) k_sumsq<<<L.nA, kThreads, 0, s>>>(P, L.itemsA);
-    if (L.nF) k_finalize<<<L.nF, kThreads, 0, s>>>(P, L.itemsF);
-    if (L.nBC) {
-        k_rms<<<L.nBC, kThreads, 0, s>>>(P, L.itemsBC);
-        k_apply<<<L.nBC, kThreads, 0, s>>>(P, L.itemsBC);
-    }
+    auto mark = [&](int k) {
+        if (ev) cudaEventRecord((cudaEvent_t)ev[k], s);
+    };
+    mark(0);
+    if (L.nA) k_sumsq<<<L.nA, kThreads, 0, s>>>(A, L.itemsA);
+    mark(1);
+    if (L.nF) k_finalize<<<L.nF, kThreads, 0, s>>>(A, L.itemsF);
+    mark(2);
+    if (L.nBC) k_rms<<<L.nBC, kThreads, 0, s>>>(A, L.itemsBC);
+    mark(3);
+    if (L.nBC) k_apply<<<L.nBC, kThreads, 0, s>>>(A, L.itemsBC);
+    mark(4);
     return (int)cudaGetLastError();
 }
 

@@ -35,13 +35,12 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Writes the descriptor, clears the scalars (the step's completion counters
 // must start at zero) and fills the three item tables of one tensor.
-__global__ void k_noalloc_setup(TensorDev td, TensorDev *dst, StepArgs args, StepArgs *args_dst, TensorScal *scal,
-                                uint2 *itemsA, uint32_t nA, uint2 *itemsF, uint32_t nF, uint2 *itemsBC, uint32_t nBC) {
+__global__ void k_noalloc_setup(TensorDev td, TensorDev *dst, TensorScal *scal, uint2 *itemsA, uint32_t nA,
+                                uint2 *itemsF, uint32_t nF, uint2 *itemsBC, uint32_t nBC) {
     const uint32_t stride = gridDim.x * blockDim.x;
     const uint32_t i0 = blockIdx.x * blockDim.x + threadIdx.x;
     if (i0 == 0) {
         *dst = td;
-        *args_dst = args;
         *scal = TensorScal{};
     }
     for (uint32_t i = i0; i < nA; i += stride) itemsA[i] = make_uint2(0, i);
@@ -126,7 +125,6 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     // ---- scratch layout inside the fixed array --------------------------------------
     size_t off = 0;
     const size_t o_scal = off;   off = align256(off + sizeof(TensorScal));
-    const size_t o_args = off;   off = align256(off + sizeof(StepArgs));
     const size_t o_tens = off;   off = align256(off + sizeof(TensorDev));
     const size_t o_iA = off;     off = align256(off + sizeof(uint2) * nA);
     const size_t o_iF = off;     off = align256(off + sizeof(uint2) * nF);
@@ -211,14 +209,14 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     a.seed_hi = (uint32_t)(seed >> 32);
 
     cudaStream_t s = (cudaStream_t)stream;
-    k_noalloc_setup<<<8, 256, 0, s>>>(td, (TensorDev *)(base + o_tens), a, (StepArgs *)(base + o_args),
-                                      (TensorScal *)(base + o_scal), (uint2 *)(base + o_iA), nA, (uint2 *)(base + o_iF),
-                                      nF, (uint2 *)(base + o_iBC), nBC);
+    k_noalloc_setup<<<8, 256, 0, s>>>(td, (TensorDev *)(base + o_tens), (TensorScal *)(base + o_scal),
+                                      (uint2 *)(base + o_iA), nA, (uint2 *)(base + o_iF), nF, (uint2 *)(base + o_iBC),
+                                      nBC);
     e = cudaGetLastError();
     if (e != cudaSuccess) return SKEW_ECUDA;
     const LaunchPlan lp{nA, nF, nBC, (const uint2 *)(base + o_iA), (const uint2 *)(base + o_iF),
                         (const uint2 *)(base + o_iBC)};
-    e = (cudaError_t)launch_phases((const StepArgs *)(base + o_args), lp, stream);
+    e = (cudaError_t)launch_phases(a, lp, stream, nullptr);
     if (e != cudaSuccess) return SKEW_ECUDA;
     return SKEW_OK;
 }

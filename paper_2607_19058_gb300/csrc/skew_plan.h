@@ -57,8 +57,7 @@ struct TensorScal {
 };
 static_assert(sizeof(TensorScal) == 64, "TensorScal layout");
 
-// Per-step parameters. skew_step writes them into a device-resident block that
-// every kernel reads, so that a captured graph of the step never changes.
+// Per-step parameters, passed by value to every kernel (a kernel parameter).
 struct StepArgs {
     const TensorDev *tensors;
     TensorScal *scal;
@@ -81,7 +80,9 @@ struct LaunchPlan {
 };
 
 // Enqueues the phases of `L` as four grouped launches (A, F, B, C) on `stream`,
-// all reading the parameter block P (device memory); returns a cudaError_t value.
-int launch_phases(const StepArgs *P, const LaunchPlan &L, void *stream);
+// each given the step parameters A by value. If `ev` is not null it holds five
+// cudaEvent_t, recorded before the first launch and after each of the four.
+// Returns a cudaError_t value.
+int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *const *ev);
 
 }  // namespace skew
