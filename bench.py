@@ -120,8 +120,8 @@ def clocks_stop(handle):
 # ---------------------------------------------------------------------------
 def byte_model(opt, n_tensors):
     """Algorithmic minimum bytes of one step and of each kernel's own traffic."""
-    N = N_mom = N_full = N_fact = N_nomom = 0
-    rc = 0
+    N = N_mom = N_full = N_fact = N_nomom = N_row = 0
+    rc = rc_row = 0
     for k in range(n_tensors):
         i = opt.info(k)
         N += i.numel
@@ -131,15 +131,19 @@ def byte_model(opt, n_tensors):
             N_nomom += i.numel
         if i.kind == 0:
             N_full += i.numel
+        elif i.rowpath:
+            N_row += i.numel
+            rc_row += i.rows + i.cols
         else:
             N_fact += i.numel
             rc += i.rows + i.cols
-    step_min = 6 * N + 8 * N_mom + 8 * N_full + 8 * rc
+    step_min = 6 * N + 8 * N_mom + 8 * N_full + 8 * (rc + rc_row)
     kernels = {
-        "step_graph": step_min,                                  # the whole step: one graph launch
-        "k_sumsq": 2 * N_fact,                                   # read G of factored matrices
-        "k_finalize": 8 * rc,                                    # R, C read + write
-        "k_rms": 2 * N + 8 * N_mom + 8 * N_full,                 # read G; M, v read + write
+        "k_sumsq": 2 * N_fact,                                   # read G of strip-path factored matrices
+        "k_rowsq": 2 * N_row + 8 * rc_row,                       # read G of row-path matrices; R read + write
+        "k_finalize": 8 * (rc + rc_row),                         # R, C read + write
+        "k_rms": 2 * (N - N_row) + 8 * N_mom + 8 * N_full,       # read G; M, v read + write
+        "k_fallback": 0,                                          # runs only when a clamp may bind
         "k_apply": 4 * N + 2 * N_nomom + 4 * N_mom + 4 * N_full,  # W r/w; G or M; v read
     }
     return dict(N=N, N_mom=N_mom, N_full=N_full, rc=rc, step_min=step_min, kernels=kernels)

@@ -132,6 +132,9 @@ typedef struct {
     int32_t vectorized; /* 1 if the 16-byte vector path serves it (after bind) */
     int64_t rows, cols, numel;
     int64_t m_offset, v_offset, r_offset, c_offset;
+    int32_t rowpath;    /* 1 if phase A runs on whole rows and sum(U^2) needs no  */
+                        /* second pass over G unless a clamp may bind (bilinear) */
+    int32_t reserved;   /* 0                                                   */
 } skew_tensor_info_t;
 
 /*
@@ -210,7 +213,8 @@ int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *ou
 /*
  * Benchmark support: launch timing. After skew_profile_begin(h, n), each of the
  * next n calls of skew_step records a CUDA event before and after each timed
- * launch it makes on the step's stream (one: the step graph; no extra
+ * launch it makes on the step's stream (six grouped launches, named by
+ * skew_kernel_name; a phase with no work times ~0; no extra
  * synchronisation). skew_profile_end(h, ms, cap, &steps, &launches)
  * synchronises, writes the durations in milliseconds row-major into
  * ms[steps][launches] (up to cap values), releases the events and stops
@@ -233,9 +237,10 @@ const char *skew_kernel_name(int32_t k);
  * workspace; this entry point instead uses a fixed scratch array compiled into
  * the library: SKEW_NOALLOC_SCRATCH_BYTES of device memory on every GPU that
  * loads the library, held until the process exits. That is enough for one
- * tensor of up to about 50,000 x 4,096 (the paper's 50,304 x 4,096 embedding
- * fits); larger tensors are rejected with SKEW_ETOOBIG before any work is
- * enqueued.
+ * tensor of up to about 50,000 x 4,096 with momentum (the paper's 50,304 x
+ * 4,096 embedding fits) or about 43,000 x 4,096 without (an expert matrix's
+ * whole-row partials take more room); larger tensors are rejected with
+ * SKEW_ETOOBIG before any work is enqueued.
  *
  * Arguments: weight / grad as in skew_param_desc_t (device, bf16, row-major);
  * ndim, rows, cols, tier, flags as in skew_param_desc_t; hp as for

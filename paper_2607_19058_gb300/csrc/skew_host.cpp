@@ -29,7 +29,9 @@ struct TPlan {
     int64_t n = 0, m = 0, numel = 0;
     int64_t moff = -1, voff = -1, roff = -1, coff = -1;  // floats into the state
     uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
-    size_t ws_rowp = 0, ws_colp = 0, ws_bsc = 0, ws_rsum = 0, ws_u2 = 0;  // bytes into the workspace
+    uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0;
+    // bytes into the workspace
+    size_t ws_rowp = 0, ws_colp = 0, ws_bsc = 0, ws_rsum = 0, ws_u2 = 0, ws_pp = 0, ws_rmin = 0, ws_fsum = 0, ws_fmin = 0;
 };
 
 thread_local std::string g_create_err;
@@ -43,9 +45,11 @@ struct skew_handle {
     skew_hparams_t hp{};
     std::vector<TPlan> t;
     size_t state_bytes = 0, ws_bytes = 0;
-    size_t ws_scal = 0, ws_err = 0, ws_tab = 0, ws_tab_end = 0;
-    size_t ws_tens = 0, ws_itemsA = 0, ws_itemsF = 0, ws_itemsBC = 0;
-    std::vector<uint2> itemsA, itemsF, itemsBC;  // per phase, tensors in order
+    size_t ws_scal = 0, ws_fb = 0, ws_err = 0, ws_tab = 0, ws_tab_end = 0;
+    size_t ws_tens = 0, ws_itemsA = 0, ws_itemsR = 0, ws_itemsF = 0, ws_itemsB = 0, ws_itemsC = 0;
+    std::vector<uint2> itemsA, itemsR, itemsF, itemsB, itemsC;  // per phase, tensors in order
+    uint32_t n_rowpath = 0;  // tensors on the row path
+    uint32_t fb_ctas = 0;    // CTAs of the row path's phase-B launch (set at bind)
     char *state = nullptr, *ws = nullptr;
     bool bound = false;
     std::string err;
@@ -57,9 +61,9 @@ struct skew_handle {
     }
 };
 
-// What the profiler times per step: the four grouped launches.
-constexpr int kProfLaunches = 4;
-const char *const kProfNames[kProfLaunches] = {"k_sumsq", "k_finalize", "k_rms", "k_apply"};
+// What the profiler times per step: the grouped launches (an empty phase times ~0).
+constexpr int kProfLaunches = kLaunches;
+const char *const kProfNames[kProfLaunches] = {"k_sumsq", "k_rowsq", "k_finalize", "k_rms", "k_fallback", "k_apply"};
 
 static int fail(skew_handle_t *h, int code, const char *fmt, ...) {
     char buf[512];
@@ -95,31 +99,21 @@ static void resolve(int ndim, int tier, int policy, uint32_t flags, TPlan &p) {
     p.decay = (tier != SKEW_TIER_ROUTER) && !(flags & SKEW_F_NO_DECAY);
 }
 
-// Tile geometry: a factored tile is (tile_rows rows) x (8*LC columns), a full
-// tile is 32 Ki flat elements.
-static void geometry(TPlan &p) {
-    if (p.kind == kKindFactored) {
-        int64_t vecs = (p.m + 7) / 8;  // 8-column groups per row
-        uint32_t lc = 1, lcl = 0;
-        while (lc < 32 && lc < vecs) {
-            lc <<= 1;
-            ++lcl;
-        }
-        p.lcl = lcl;
-        p.strips = (uint32_t)((p.m + 8 * lc - 1) / (8 * lc));
-        p.tile_rows = (uint32_t)(kVecPerThread * (kThreads / lc));
-        p.rowtiles = (uint32_t)((p.n + p.tile_rows - 1) / p.tile_rows);
-        p.ntiles = p.strips * p.rowtiles;
-        p.nfr = (uint32_t)((p.n + kFinChunk - 1) / kFinChunk);
-        p.nfc = (uint32_t)((p.m + kFinChunk - 1) / kFinChunk);
-    } else {
-        p.lcl = 0;
-        p.strips = 1;
-        p.tile_rows = 0;
-        p.rowtiles = (uint32_t)((p.numel + kFlatTileElems - 1) / kFlatTileElems);
-        p.ntiles = p.rowtiles;
-        p.nfr = p.nfc = 0;
-    }
+// Tile geometry (plan_geometry): strip tiles of (tile_rows rows) x (8*LC
+// columns) or flat tiles of 64 Ki elements, and for the row path whole-row tiles.
+static void geometry(TPlan &p, bool wg_aligned) {
+    const TileGeom g = plan_geometry(p.kind, p.momentum, wg_aligned, p.n, p.m, p.numel);
+    p.lcl = g.lcl;
+    p.strips = g.strips;
+    p.rowtiles = g.rowtiles;
+    p.tile_rows = g.tile_rows;
+    p.ntiles = g.ntiles;
+    p.nfr = g.nfr;
+    p.nfc = g.nfc;
+    p.rowpath = g.rowpath;
+    p.cr = g.cr;
+    p.rt_rows = g.rt_rows;
+    p.rtiles = g.rtiles;
 }
 
 extern "C" {
@@ -165,7 +159,12 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
         if (p.n > (int64_t(1) << 62) / p.m) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: too many elements", k); }
         p.numel = p.n * p.m;
         resolve(d.ndim, d.tier, H.policy, d.flags, p);
-        geometry(p);
+        // tiles are indexed with 32 bits: at most 2^31 per tensor
+        const int64_t tiles64 = p.kind == kKindFactored ? ((p.m + 255) / 256) * ((p.n + 255) / 256)
+                                                        : (p.numel + kFlatTileElems - 1) / kFlatTileElems;
+        if (tiles64 > (int64_t(1) << 31)) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: too many elements", k); }
+        geometry(p, (((uintptr_t)d.weight | (uintptr_t)d.grad) & 15) == 0);
+        h->n_rowpath += p.rowpath;
     }
 
     // State layout (fp32 offsets): [momentum arrays][full v arrays][R arrays][C arrays].
@@ -190,38 +189,57 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
         for (int q = 0; q < n_params; ++q) {
             const TPlan &p = h->t[q];
             if (p.kind == kKindFactored) {
-                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(q, i));
+                if (p.rowpath)
+                    for (uint32_t i = 0; i < p.rtiles; ++i) h->itemsR.push_back(make_uint2(q, i));
+                else
+                    for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(q, i));
                 for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(q, i));
             }
-            for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsBC.push_back(make_uint2(q, i));
+            if (!p.rowpath)
+                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsB.push_back(make_uint2(q, i));
+            for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsC.push_back(make_uint2(q, i));
         }
     } catch (...) {
         delete h;
         return fail(nullptr, SKEW_ENOMEM, "out of host memory");
     }
 
-    // Workspace layout (bytes, 256-aligned regions).
+    // Workspace layout (bytes, 256-aligned regions). The scalars and the row
+    // path's phase-B queue ([count][tensor ids]) are zeroed every step.
     size_t w = 0;
     h->ws_scal = w;
     w = align_up(w + sizeof(TensorScal) * n_params, 256);
+    h->ws_fb = w;
+    w = align_up(w + 4 * (size_t(h->n_rowpath) + 1), 256);
     h->ws_err = w;
     w = align_up(w + 16, 256);
     h->ws_tab = w;
     h->ws_tens = w;
     w = align_up(w + sizeof(TensorDev) * n_params, 256);
-    h->ws_itemsA = w;
-    w = align_up(w + sizeof(uint2) * h->itemsA.size(), 256);
-    h->ws_itemsF = w;
-    w = align_up(w + sizeof(uint2) * h->itemsF.size(), 256);
-    h->ws_itemsBC = w;
-    w = align_up(w + sizeof(uint2) * h->itemsBC.size(), 256);
+    auto table = [&](size_t &at, const std::vector<uint2> &v) {
+        at = w;
+        w = align_up(w + sizeof(uint2) * v.size(), 256);
+    };
+    table(h->ws_itemsA, h->itemsA);
+    table(h->ws_itemsR, h->itemsR);
+    table(h->ws_itemsF, h->itemsF);
+    table(h->ws_itemsB, h->itemsB);
+    table(h->ws_itemsC, h->itemsC);
     h->ws_tab_end = w;
     for (auto &p : h->t) {
-        if (p.kind == kKindFactored) {
+        if (p.kind == kKindFactored && !p.rowpath) {
             p.ws_rowp = w; w = align_up(w + 4 * size_t(p.strips) * p.n, 256);
             p.ws_colp = w; w = align_up(w + 4 * size_t(p.rowtiles) * p.m, 256);
             p.ws_bsc = w;  w = align_up(w + 4 * size_t(p.m), 256);
             p.ws_rsum = w; w = align_up(w + 8 * size_t(p.nfr), 256);
+        } else if (p.kind == kKindFactored) {
+            p.ws_colp = w; w = align_up(w + 4 * size_t(p.rtiles) * p.m, 256);
+            p.ws_pp = w;   w = align_up(w + 8 * size_t(p.rtiles) * p.m, 256);
+            p.ws_bsc = w;  w = align_up(w + 4 * size_t(p.m), 256);
+            p.ws_rsum = w; w = align_up(w + 8 * size_t(p.rtiles), 256);
+            p.ws_rmin = w; w = align_up(w + 4 * size_t(p.rtiles), 256);
+            p.ws_fsum = w; w = align_up(w + 8 * size_t(p.nfc), 256);
+            p.ws_fmin = w; w = align_up(w + 4 * size_t(p.nfc), 256);
         }
         p.ws_u2 = w;
         w = align_up(w + 8 * size_t(p.ntiles), 256);
@@ -244,7 +262,8 @@ int32_t skew_num_tensors(const skew_handle_t *h) { return h ? (int32_t)h->t.size
 
 int64_t skew_launches_per_step(const skew_handle_t *h) {
     if (!h) return 0;
-    return int64_t(!h->itemsA.empty()) + int64_t(!h->itemsF.empty()) + 2 * int64_t(!h->itemsBC.empty());
+    return int64_t(!h->itemsA.empty()) + int64_t(!h->itemsR.empty()) + int64_t(!h->itemsF.empty()) +
+           int64_t(!h->itemsB.empty()) + int64_t(h->n_rowpath > 0) + int64_t(!h->itemsC.empty());
 }
 
 const char *skew_last_error(const skew_handle_t *h) { return h ? h->err.c_str() : g_create_err.c_str(); }
@@ -264,6 +283,8 @@ int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *ou
     out->v_offset = p.voff;
     out->r_offset = p.roff;
     out->c_offset = p.coff;
+    out->rowpath = (int32_t)p.rowpath;
+    out->reserved = 0;
     return SKEW_OK;
 }
 
@@ -298,10 +319,15 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.v = p.voff >= 0 ? sf + p.voff : nullptr;
         T.R = p.roff >= 0 ? sf + p.roff : nullptr;
         T.C = p.coff >= 0 ? sf + p.coff : nullptr;
-        T.rowp = p.kind == kKindFactored ? (float *)(h->ws + p.ws_rowp) : nullptr;
-        T.colp = p.kind == kKindFactored ? (float *)(h->ws + p.ws_colp) : nullptr;
-        T.bsc = p.kind == kKindFactored ? (float *)(h->ws + p.ws_bsc) : nullptr;
-        T.rsum = p.kind == kKindFactored ? (double *)(h->ws + p.ws_rsum) : nullptr;
+        const bool fact = p.kind == kKindFactored, row = fact && p.rowpath;
+        T.rowp = fact && !row ? (float *)(h->ws + p.ws_rowp) : nullptr;
+        T.colp = fact ? (float *)(h->ws + p.ws_colp) : nullptr;
+        T.bsc = fact ? (float *)(h->ws + p.ws_bsc) : nullptr;
+        T.rsum = fact ? (double *)(h->ws + p.ws_rsum) : nullptr;
+        T.pp = row ? (double *)(h->ws + p.ws_pp) : nullptr;
+        T.rmin = row ? (float *)(h->ws + p.ws_rmin) : nullptr;
+        T.fsum = row ? (double *)(h->ws + p.ws_fsum) : nullptr;
+        T.fmin = row ? (float *)(h->ws + p.ws_fmin) : nullptr;
         T.u2 = (float2 *)(h->ws + p.ws_u2);
         T.n = p.n;
         T.m = p.m;
@@ -324,13 +350,19 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.ntiles = p.ntiles;
         T.nfr = p.nfr;
         T.nfc = p.nfc;
+        T.rowpath = p.rowpath;
+        T.cr = p.cr;
+        T.rt_rows = p.rt_rows;
+        T.rtiles = p.rtiles;
     }
     auto put = [&](size_t at, const std::vector<uint2> &v) {
         if (!v.empty()) std::memcpy(img.data() + (at - h->ws_tab), v.data(), v.size() * sizeof(uint2));
     };
     put(h->ws_itemsA, h->itemsA);
+    put(h->ws_itemsR, h->itemsR);
     put(h->ws_itemsF, h->itemsF);
-    put(h->ws_itemsBC, h->itemsBC);
+    put(h->ws_itemsB, h->itemsB);
+    put(h->ws_itemsC, h->itemsC);
 
     cudaError_t e;
     if (!img.empty()) {
@@ -350,6 +382,11 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
     }
     e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(h, e, "bind");
+    // the row path's phase-B launch: two CTAs per SM split a queued tensor's tiles
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+        return cuda_fail(h, e, "device query");
+    h->fb_ctas = (uint32_t)(2 * (sms > 0 ? sms : 1));
 
     h->bound = true;
     return SKEW_OK;
@@ -370,6 +407,8 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
     StepArgs a{};
     a.tensors = reinterpret_cast<const TensorDev *>(h->ws + h->ws_tens);
     a.scal = reinterpret_cast<TensorScal *>(h->ws + h->ws_scal);
+    a.err = reinterpret_cast<uint32_t *>(h->ws + h->ws_err);
+    a.fb = reinterpret_cast<uint32_t *>(h->ws + h->ws_fb);
     a.b1 = H.beta1;
     a.b2 = H.beta2;
     a.c1 = (float)(1.0 - (double)H.beta1);
@@ -389,12 +428,13 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
         ev = h->prof_ev.data() + size_t(h->prof_used) * (kProfLaunches + 1);
         ++h->prof_used;
     }
-    cudaError_t e = cudaMemsetAsync(h->ws + h->ws_scal, 0, sizeof(TensorScal) * h->t.size(), s);
+    cudaError_t e = cudaMemsetAsync(h->ws + h->ws_scal, 0, h->ws_fb + 4 - h->ws_scal, s);
     if (e != cudaSuccess) return cuda_fail(h, e, "reset of per-step scalars");
-    const LaunchPlan L{(uint32_t)h->itemsA.size(), (uint32_t)h->itemsF.size(), (uint32_t)h->itemsBC.size(),
-                       reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsA),
-                       reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsF),
-                       reinterpret_cast<const uint2 *>(h->ws + h->ws_itemsBC)};
+    auto items = [&](size_t at) { return reinterpret_cast<const uint2 *>(h->ws + at); };
+    const LaunchPlan L{(uint32_t)h->itemsA.size(), (uint32_t)h->itemsR.size(), (uint32_t)h->itemsF.size(),
+                       (uint32_t)h->itemsB.size(), h->n_rowpath ? h->fb_ctas : 0u, (uint32_t)h->itemsC.size(),
+                       items(h->ws_itemsA), items(h->ws_itemsR), items(h->ws_itemsF), items(h->ws_itemsB),
+                       items(h->ws_itemsC)};
     e = (cudaError_t)launch_phases(a, L, s, reinterpret_cast<void *const *>(ev));
     if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
     return SKEW_OK;

@@ -460,11 +460,398 @@ __device__ void sumsq_tile(const TensorDev &T, uint32_t tile, Smem &sm, const Po
 }
 
 // ---------------------------------------------------------------------------
+// Row path, phase A (k_rowsq): whole-row tiles of a momentum-free factored
+// matrix. With a_i = sqrt(Rbar / R_i) and b_j = 1/sqrt(C_j), and no element at
+// the clamp, sum_ij (g_ij a_i b_j)^2 = Rbar * sum_j (1 / C_j) * P_j with
+// P_j = sum_i g_ij^2 / R_i. A tile holds whole rows, so it forms R_i (Eq. 1)
+// itself and adds g_ij^2 / R_i into per-column partials of P; the column
+// finalize then gives C_j and sum(U^2) without phase B re-reading G.
+// Each chunk (kRowChunkBytes of consecutive rows, contiguous in memory) is
+// brought to shared memory by one bulk copy completing on an mbarrier; the
+// CTA keeps kRowStages chunks in flight.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(b)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(b)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Polls of one mbarrier wait before it gives up (each poll may suspend the
+// thread for a short hardware-defined time): a copy that never lands ends the
+// tile with a status word instead of hanging the GPU.
+constexpr uint32_t kMbarPolls = 1u << 20;
+
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
+    for (uint32_t i = 0; i < kMbarPolls; ++i)
+        if (mbar_try_wait(b, parity)) return true;
+    return false;
+}
+
+// Bulk copy global -> shared of `bytes` (multiple of 16, both ends 16-byte
+// aligned), completing on mbarrier `bar`, with an L2 eviction policy.
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar, uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
+        : "memory");
+}
+
+// Orders this thread's earlier generic-proxy accesses of shared memory before
+// its later async-proxy (bulk copy) accesses.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+
+struct RowSmem {
+    uint4 buf[kRowStages][kRowChunkBytes / 16];  // the chunk ring (first member: 16-byte aligned)
+    uint64_t full[kRowStages];                   // one mbarrier per ring slot
+    float part[kThreads / 32][8];                // per-warp row partial sums of the chunk
+    float inv[8];                                // 1 / R_i of the chunk's rows (0: no contribution)
+    int fail;
+};
+
+// Rows `i` of chunk `c` of row tile `tile`: [i0, i0 + rows).
+struct RowChunk {
+    int64_t i0;
+    uint32_t rows;
+};
+
+__device__ __forceinline__ RowChunk row_chunk(const TensorDev &T, uint32_t tile, uint32_t c) {
+    const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * T.cr;
+    const int64_t left = T.n - i0;
+    return RowChunk{i0, left <= 0 ? 0u : (uint32_t)min(left, (int64_t)T.cr)};
+}
+
+// Sum over a warp of K per-lane values, transposed: lane L ends with the total
+// of value j(L) (K = 8: j = 4*b4 + 2*b3 + b2 of L's bits; K = 4: j = 2*b4 + b3),
+// held by the lanes whose low bits (3 for K = 8, 2 + 1 for K = 4) are zero.
+template <int K>
+__device__ __forceinline__ float warp_sum_transposed(const float (&x)[K], int &j) {
+    const uint32_t ln = threadIdx.x & 31;
+    const bool b4 = ln & 16, b3 = ln & 8, b2 = ln & 4;
+    if constexpr (K == 8) {
+        float v4[4], v2[2];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float keep = b4 ? x[q + 4] : x[q], send = b4 ? x[q] : x[q + 4];
+            v4[q] = keep + __shfl_xor_sync(kAll, send, 16);
+        }
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const float keep = b3 ? v4[q + 2] : v4[q], send = b3 ? v4[q] : v4[q + 2];
+            v2[q] = keep + __shfl_xor_sync(kAll, send, 8);
+        }
+        float v1 = (b2 ? v2[1] : v2[0]) + __shfl_xor_sync(kAll, b2 ? v2[0] : v2[1], 4);
+        v1 += __shfl_xor_sync(kAll, v1, 2);
+        v1 += __shfl_xor_sync(kAll, v1, 1);
+        j = (b4 ? 4 : 0) + (b3 ? 2 : 0) + (b2 ? 1 : 0);
+        return v1;
+    } else {
+        float v2[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const float keep = b4 ? x[q + 2] : x[q], send = b4 ? x[q] : x[q + 2];
+            v2[q] = keep + __shfl_xor_sync(kAll, send, 16);
+        }
+        float v1 = (b3 ? v2[1] : v2[0]) + __shfl_xor_sync(kAll, b3 ? v2[0] : v2[1], 8);
+        v1 += __shfl_xor_sync(kAll, v1, 4);
+        v1 += __shfl_xor_sync(kAll, v1, 2);
+        v1 += __shfl_xor_sync(kAll, v1, 1);
+        j = (b4 ? 2 : 0) + (b3 ? 1 : 0);
+        return v1;
+    }
+}
+
+// Issues the bulk copy of chunk c of the tile into ring slot c % kRowStages.
+__device__ __forceinline__ void row_issue(const TensorDev &T, uint32_t tile, uint32_t c, RowSmem &sm, uint64_t pol) {
+    const RowChunk ch = row_chunk(T, tile, c);
+    const uint32_t bytes = ch.rows * (uint32_t)T.m * 2u;
+    const int st = c % kRowStages;
+    mbar_expect_tx(&sm.full[st], bytes);
+    bulk_g2s(sm.buf[st], T.g + ch.i0 * T.m, bytes, &sm.full[st], pol);
+}
+
+// NV 16-byte vectors per thread per row (m = 2048 * NV), CR = 8 / NV rows per chunk.
+template <int NV>
+__device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S, uint32_t tile, RowSmem &sm) {
+    constexpr int CR = 8 / NV;
+    constexpr int V = kThreads * NV;  // vectors per row
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    const uint32_t nch = (uint32_t)min((int64_t)kRowChunks, (T.n - int64_t(tile) * T.rt_rows + T.cr - 1) / T.cr);
+    if (threadIdx.x == 0) {
+        for (int st = 0; st < kRowStages; ++st) mbar_init(&sm.full[st], 1);
+        fence_mbar_init();
+        sm.fail = 0;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+        for (uint32_t c = 0; c < nch && c < (uint32_t)kRowStages; ++c) row_issue(T, tile, c, sm, pol);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const float b2 = A.b2, c2 = A.c2, fm = (float)T.m;
+    float cs[NV][8], ph[NV][8], pl[NV][8];
+#pragma unroll
+    for (int v = 0; v < NV; ++v)
+#pragma unroll
+        for (int c = 0; c < 8; ++c) cs[v][c] = ph[v][c] = pl[v][c] = 0.f;
+    double rsum = 0.0;                       // threads < CR: sum of this lane's rows' R
+    float rmin = __int_as_float(0x7F800000);  // threads < CR: smallest positive R of this lane's rows
+    bool zero_row = false;
+
+    uint32_t c = 0;
+    for (; c < nch; ++c) {
+        const int st = c % kRowStages;
+        const uint32_t par = (c / kRowStages) & 1u;
+        const RowChunk ch = row_chunk(T, tile, c);
+        float rp = 0.f;
+        if (tid < (int)ch.rows) rp = __ldcg(T.R + ch.i0 + tid);
+        const bool ok = mbar_wait(&sm.full[st], par);
+        const uint4 *buf = sm.buf[st];
+        // pass 1: row sums and column sums of g^2
+        float rs[CR];
+#pragma unroll
+        for (int r = 0; r < CR; ++r) {
+            rs[r] = 0.f;
+            if (r < (int)ch.rows) {
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    float g[8];
+                    unpack_bf8(buf[r * V + v * kThreads + tid], g);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        const float q = g[k] * g[k];
+                        cs[v][k] += q;
+                        rs[r] += q;
+                    }
+                }
+            }
+        }
+        int j;
+        const float tot = warp_sum_transposed<CR>(rs, j);
+        if ((lane & (CR == 8 ? 3 : 7)) == 0) sm.part[warp][j] = tot;
+        if (__syncthreads_or(!ok)) break;  // every slot before this one has landed
+        // slot of chunk c - 1 is free (its pass 2 preceded this barrier): refill it
+        if (tid == 0 && c >= 1 && c - 1 + kRowStages < nch) {
+            fence_proxy_async_smem();
+            row_issue(T, tile, c - 1 + kRowStages, sm, pol);
+        }
+        if (tid < (int)ch.rows) {
+            float sum = 0.f;
+#pragma unroll
+            for (int w = 0; w < kThreads / 32; ++w) sum += sm.part[w][tid];
+            const float mean = __fdiv_rn(sum, fm);
+            const float Rn = fmaf(b2, rp, c2 * mean);
+            T.R[ch.i0 + tid] = Rn;
+            rsum += (double)Rn;
+            float inv = 0.f;
+            if (Rn > 0.f && Rn < __int_as_float(0x7F800000)) {
+                rmin = fminf(rmin, Rn);
+                inv = __frcp_rn(Rn);
+            } else if (!(Rn == 0.f && sum == 0.f)) {
+                zero_row = true;  // content in a row with R_i == 0, or a non-finite R_i
+            }
+            sm.inv[tid] = inv;
+        }
+        __syncthreads();
+        // pass 2: P_j += g^2 / R_i, a chunk sum per column folded into (hi, lo)
+        float t[NV][8];
+#pragma unroll
+        for (int v = 0; v < NV; ++v)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) t[v][k] = 0.f;
+#pragma unroll
+        for (int r = 0; r < CR; ++r) {
+            if (r < (int)ch.rows) {
+                const float iv = sm.inv[r];
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    float g[8];
+                    unpack_bf8(buf[r * V + v * kThreads + tid], g);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) t[v][k] = fmaf(g[k] * g[k], iv, t[v][k]);
+                }
+            }
+        }
+#pragma unroll
+        for (int v = 0; v < NV; ++v)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                float s2, e;
+                two_sum(ph[v][k], t[v][k], s2, e);
+                ph[v][k] = s2;
+                pl[v][k] += e;
+            }
+    }
+    if (c < nch) {
+        // A chunk did not land in time: record it, give the copies in flight
+        // (chunks c .. issued) one more bounded wait each, and drop the tile.
+        // Issued so far: chunks [0, kRowStages) by the prologue and chunk k - 1 +
+        // kRowStages at each iteration k in [1, c); chunks before c have landed.
+        if (tid == 0) {
+            atomicOr(A.err, 2u);
+            const uint32_t issued_end = min(nch, c == 0 ? (uint32_t)kRowStages : c + kRowStages - 1);
+            for (uint32_t k = c; k < issued_end; ++k) (void)mbar_wait(&sm.full[k % kRowStages], (k / kRowStages) & 1u);
+        }
+        return;
+    }
+    // per-tile partials: column sums of g^2 and of g^2 / R_i, the tile's sum and
+    // smallest positive R
+    const int64_t base = int64_t(tile) * T.m;
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+        const int64_t col = 8 * int64_t(v * kThreads + tid);
+        float4 *cp4 = reinterpret_cast<float4 *>(T.colp + base + col);
+        cp4[0] = make_float4(cs[v][0], cs[v][1], cs[v][2], cs[v][3]);
+        cp4[1] = make_float4(cs[v][4], cs[v][5], cs[v][6], cs[v][7]);
+        double2 *pp2 = reinterpret_cast<double2 *>(T.pp + base + col);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            pp2[k] = make_double2((double)ph[v][2 * k] + (double)pl[v][2 * k],
+                                  (double)ph[v][2 * k + 1] + (double)pl[v][2 * k + 1]);
+    }
+    if (zero_row) atomicOr(&S.zflag, 1u);
+    if (warp == 0) {
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            rsum += __shfl_xor_sync(kAll, rsum, o);
+            rmin = fminf(rmin, __shfl_xor_sync(kAll, rmin, o));
+        }
+        if (lane == 0) {
+            T.rsum[tile] = rsum;
+            T.rmin[tile] = rmin;
+        }
+    }
+}
+
+// mean(R) and its [1, 2) mantissa / exponent split (used by the row scales).
+__device__ void set_rbar(TensorScal &S, double rbar) {
+    S.rbar = rbar;
+    if (rbar > 0.0) {
+        int e;
+        const double fr = frexp(rbar, &e);  // rbar = fr * 2^e, fr in [0.5, 1)
+        S.rbar_s = (float)(2.0 * fr);       // in [1, 2]
+        S.rbar_e = 1 - e;                   // rbar * 2^(1-e) = 2 fr
+    } else {
+        S.rbar_s = 0.f;
+        S.rbar_e = 0;
+    }
+}
+
+// From s = sum of (U / coef)^2: sum(U^2), RMS(U), the clip factor
+// kappa = 1 / max(1, RMS / d) (Sec. 3 update clipping) and lr * kappa * coef.
+__device__ void set_clip(const StepArgs &A, const TensorDev &T, TensorScal &S, double s) {
+    const double coef = T.momentum ? A.coef_mom : A.coef_plain;
+    const double su2 = s * coef * coef;
+    const double rms = sqrt(su2 / (double)T.numel);
+    const double kappa = 1.0 / fmax(1.0, rms / (double)A.clip_d);
+    S.sumsq = su2;
+    S.rms = rms;
+    S.kappa = kappa;
+    S.coefC = (float)((double)A.lr * kappa * coef);
+}
+
+// Row path, finalize item `local` (kFinChunk columns): C_j, 1/sqrt(C_j) and the
+// chunk's sum of P_j / C_j. The last item of the tensor forms mean(R) and, when
+// no element can reach the clamp (max_i a_i^2 * max_j b_j^2 <= 1/eps over rows and
+// columns that hold gradient), sum(U^2) = coef^2 * mean(R) * sum_j P_j / C_j and
+// the clip factor; otherwise it queues the tensor for phase B.
+__device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm) {
+    const TensorDev &T = A.tensors[t];
+    TensorScal &S = A.scal[t];
+    const float inf = __int_as_float(0x7F800000);
+    const int64_t j = int64_t(local) * kFinChunk + threadIdx.x;
+    double contrib = 0.0;
+    float cmin = inf;
+    if (threadIdx.x < kFinChunk && j < T.m) {
+        float cs = 0.f;
+        double P = 0.0;
+        for (uint32_t r = 0; r < T.rtiles; ++r) {
+            cs += __ldcg(T.colp + int64_t(r) * T.m + j);
+            P += __ldcg(T.pp + int64_t(r) * T.m + j);
+        }
+        const float mean = __fdiv_rn(cs, (float)T.n);
+        const float Cn = fmaf(A.b2, T.C[j], A.c2 * mean);
+        T.C[j] = Cn;
+        T.bsc[j] = __frsqrt_rn(Cn);
+        if (P > 0.0) {
+            if (Cn > 0.f && Cn < inf) {
+                contrib = P / (double)Cn;
+                cmin = Cn;
+            } else {
+                atomicOr(&S.zflag, 1u);  // gradient in a column whose C_j is 0 or not finite
+            }
+        } else if (!(P == 0.0)) {
+            atomicOr(&S.zflag, 1u);  // NaN
+        }
+    }
+    contrib = block_sum_d(contrib, sm.redd);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) cmin = fminf(cmin, __shfl_xor_sync(kAll, cmin, o));
+    if ((threadIdx.x & 31) == 0) sm.red2[threadIdx.x >> 5].x = cmin;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 0; w < kThreads / 32; ++w) cmin = fminf(cmin, sm.red2[w].x);
+        T.fsum[local] = contrib;
+        T.fmin[local] = cmin;
+        sm.last = (atom_add_acq_rel(&S.cntF, 1u) == T.nfc - 1);
+    }
+    __syncthreads();
+    if (sm.last && threadIdx.x == 0) {
+        double rs = 0.0, fs = 0.0;
+        float rmn = inf, cmn = inf;
+        for (uint32_t r = 0; r < T.rtiles; ++r) {
+            rs += __ldcg(T.rsum + r);
+            rmn = fminf(rmn, __ldcg(T.rmin + r));
+        }
+        for (uint32_t f = 0; f < T.nfc; ++f) {
+            fs += __ldcg(T.fsum + f);
+            cmn = fminf(cmn, __ldcg(T.fmin + f));
+        }
+        const double rbar = rs / (double)T.n;
+        set_rbar(S, rbar);
+        const double a2 = rmn < inf ? rbar / (double)rmn : 0.0;  // max_i a_i^2 over rows with R_i > 0
+        const double b2 = cmn < inf ? 1.0 / (double)cmn : 0.0;   // max_j b_j^2 over columns holding gradient
+        const double ce2 = (double)A.ce * (double)A.ce;
+        if (__ldcg(&S.zflag) == 0u && a2 * b2 <= ce2 * (1.0 - 1e-6)) {
+            set_clip(A, T, S, fs * rbar);
+        } else {
+            S.fallback = 1u;
+            const uint32_t q = atomicAdd(A.fb, 1u);
+            A.fb[1 + q] = t;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Phase F: factor EMAs, 1/sqrt(C_j), mean(R) (Eq. 1).
 // ---------------------------------------------------------------------------
 __device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm) {
     const TensorDev &T = A.tensors[t];
     TensorScal &S = A.scal[t];
+    if (T.rowpath) {
+        phase_F_row(A, t, local, sm);
+        return;
+    }
     if (local < T.nfr) {
         const int64_t i = int64_t(local) * kFinChunk + threadIdx.x;
         double rd = 0.0;
@@ -496,17 +883,7 @@ __device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm)
     if (sm.last && threadIdx.x == 0) {
         double s = 0.0;
         for (uint32_t f = 0; f < T.nfr; ++f) s += __ldcg(T.rsum + f);
-        const double rbar = s / (double)T.n;
-        S.rbar = rbar;
-        if (rbar > 0.0) {
-            int e;
-            const double fr = frexp(rbar, &e);  // rbar = fr * 2^e, fr in [0.5, 1)
-            S.rbar_s = (float)(2.0 * fr);       // in [1, 2]
-            S.rbar_e = 1 - e;                   // rbar * 2^(1-e) = 2 fr
-        } else {
-            S.rbar_s = 0.f;
-            S.rbar_e = 0;
-        }
+        set_rbar(S, s / (double)T.n);
     }
 }
 
@@ -652,16 +1029,7 @@ __device__ void phase_B(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm,
         s += (double)p.x + (double)p.y;
     }
     s = block_sum_d(s, sm.redd);
-    if (threadIdx.x == 0) {
-        const double coef = T.momentum ? A.coef_mom : A.coef_plain;
-        const double su2 = s * coef * coef;
-        const double rms = sqrt(su2 / (double)T.numel);
-        const double kappa = 1.0 / fmax(1.0, rms / (double)A.clip_d);
-        S.sumsq = su2;
-        S.rms = rms;
-        S.kappa = kappa;
-        S.coefC = (float)((double)A.lr * kappa * coef);
-    }
+    if (threadIdx.x == 0) set_clip(A, T, S, s);
 }
 
 // ---------------------------------------------------------------------------
@@ -829,6 +1197,36 @@ __global__ void __launch_bounds__(kThreads, SKEW_MINB_SUMSQ)
         sumsq_tile<false>(T, it.y, sm, pol);
 }
 
+// Row path, phase A: one row tile per CTA (dynamic shared memory: RowSmem).
+__global__ void __launch_bounds__(kThreads, 2) k_rowsq(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
+    extern __shared__ uint4 dyn_smem[];
+    RowSmem &sm = *reinterpret_cast<RowSmem *>(dyn_smem);
+    const uint2 it = items[blockIdx.x];
+    const TensorDev &T = A.tensors[it.x];
+    if (T.m == 4096)
+        rowsq_tile<2>(A, T, A.scal[it.x], it.y, sm);
+    else
+        rowsq_tile<1>(A, T, A.scal[it.x], it.y, sm);
+}
+
+// Phase B of the row-path tensors whose finalize found that a clamp may bind
+// (queued in A.fb): the CTAs of this grid split each such tensor's tiles.
+__global__ void __launch_bounds__(kThreads, 2) k_fallback(const __grid_constant__ StepArgs A) {
+    __shared__ Smem sm;
+    __shared__ Meta meta;
+    const Pol pol;
+    const uint32_t cnt = __ldcg(A.fb);
+    for (uint32_t q = 0; q < cnt; ++q) {
+        const uint32_t t = __ldcg(A.fb + 1 + q);
+        const TensorDev &T = A.tensors[t];
+        for (uint32_t tile = blockIdx.x; tile < T.ntiles; tile += gridDim.x) {
+            (void)fill_meta(T, A.scal[t], tile, A.ce, meta);
+            phase_B(A, t, tile, sm, meta, pol);
+            __syncthreads();
+        }
+    }
+}
+
 __global__ void __launch_bounds__(kThreads) k_finalize(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
     __shared__ Smem sm;
     const uint2 it = items[blockIdx.x];
@@ -891,12 +1289,20 @@ int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *co
     mark(0);
     if (L.nA) k_sumsq<<<L.nA, kThreads, 0, s>>>(A, L.itemsA);
     mark(1);
-    if (L.nF) k_finalize<<<L.nF, kThreads, 0, s>>>(A, L.itemsF);
+    if (L.nR) {
+        const cudaError_t e = cudaFuncSetAttribute(k_rowsq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RowSmem));
+        if (e != cudaSuccess) return (int)e;
+        k_rowsq<<<L.nR, kThreads, sizeof(RowSmem), s>>>(A, L.itemsR);
+    }
     mark(2);
-    if (L.nBC) k_rms<<<L.nBC, kThreads, 0, s>>>(A, L.itemsBC);
+    if (L.nF) k_finalize<<<L.nF, kThreads, 0, s>>>(A, L.itemsF);
     mark(3);
-    if (L.nBC) k_apply<<<L.nBC, kThreads, 0, s>>>(A, L.itemsBC);
+    if (L.nB) k_rms<<<L.nB, kThreads, 0, s>>>(A, L.itemsB);
     mark(4);
+    if (L.nFB) k_fallback<<<L.nFB, kThreads, 0, s>>>(A);
+    mark(5);
+    if (L.nC) k_apply<<<L.nC, kThreads, 0, s>>>(A, L.itemsC);
+    mark(6);
     return (int)cudaGetLastError();
 }
 

@@ -9,7 +9,7 @@
 // start-up. For them this entry point keeps the scratch in a fixed array
 // compiled into the library (g_scratch below, SKEW_NOALLOC_SCRATCH_BYTES bytes
 // in the device memory of every GPU that loads the library, held until the
-// process exits) and launches the same four kernels as skew_step.
+// process exits) and launches the same kernels as skew_step.
 //
 // The array's address is a device address that host code cannot name
 // directly: the host-side symbol is only a stand-in. It is looked up once per
@@ -33,19 +33,34 @@ std::mutex g_mu;
 unsigned char *g_scratch_ptr[kMaxDevices] = {};
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Writes the descriptor, clears the scalars (the step's completion counters
-// must start at zero) and fills the three item tables of one tensor.
-__global__ void k_noalloc_setup(TensorDev td, TensorDev *dst, TensorScal *scal, uint2 *itemsA, uint32_t nA,
-                                uint2 *itemsF, uint32_t nF, uint2 *itemsBC, uint32_t nBC) {
+struct SetupTables {
+    uint2 *A;
+    uint32_t nA;
+    uint2 *R;
+    uint32_t nR;
+    uint2 *F;
+    uint32_t nF;
+    uint2 *B;
+    uint32_t nB;
+    uint2 *C;
+    uint32_t nC;
+};
+
+// Writes the descriptor, clears the scalars and the phase-B queue (the step's
+// completion counters must start at zero) and fills the item tables of one tensor.
+__global__ void k_noalloc_setup(TensorDev td, TensorDev *dst, TensorScal *scal, uint32_t *fb, SetupTables tb) {
     const uint32_t stride = gridDim.x * blockDim.x;
     const uint32_t i0 = blockIdx.x * blockDim.x + threadIdx.x;
     if (i0 == 0) {
         *dst = td;
         *scal = TensorScal{};
+        fb[0] = 0u;
     }
-    for (uint32_t i = i0; i < nA; i += stride) itemsA[i] = make_uint2(0, i);
-    for (uint32_t i = i0; i < nF; i += stride) itemsF[i] = make_uint2(0, i);
-    for (uint32_t i = i0; i < nBC; i += stride) itemsBC[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < tb.nA; i += stride) tb.A[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < tb.nR; i += stride) tb.R[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < tb.nF; i += stride) tb.F[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < tb.nB; i += stride) tb.B[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < tb.nC; i += stride) tb.C[i] = make_uint2(0, i);
 }
 
 }  // namespace
@@ -102,41 +117,43 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     float *R = kind == kKindFactored ? after_m : nullptr;
     float *Cc = kind == kKindFactored ? after_m + n : nullptr;
 
-    // ---- tile geometry (the planner's: 8-element vectors, 16 rows per thread) -------
-    uint32_t lcl = 0, strips = 1, rowtiles, tile_rows = 0, ntiles, nfr = 0, nfc = 0;
-    if (kind == kKindFactored) {
-        const int64_t vecs = (m + 7) / 8;
-        uint32_t lc = 1;
-        while (lc < 32 && lc < vecs) {
-            lc <<= 1;
-            ++lcl;
-        }
-        strips = (uint32_t)((m + 8 * lc - 1) / (8 * lc));
-        tile_rows = (uint32_t)(kVecPerThread * (kThreads / lc));
-        rowtiles = (uint32_t)((n + tile_rows - 1) / tile_rows);
-        nfr = (uint32_t)((n + kFinChunk - 1) / kFinChunk);
-        nfc = (uint32_t)((m + kFinChunk - 1) / kFinChunk);
-    } else {
-        rowtiles = (uint32_t)((numel + kFlatTileElems - 1) / kFlatTileElems);
-    }
-    ntiles = strips * rowtiles;
-    const uint32_t nA = kind == kKindFactored ? ntiles : 0, nF = nfr + nfc, nBC = ntiles;
+    // ---- tile geometry and item counts (the planner's, plan_geometry) ---------------
+    const bool wg_aligned = (((uintptr_t)weight | (uintptr_t)grad) & 15) == 0;
+    const int64_t tiles64 = kind == kKindFactored ? ((m + 255) / 256) * ((n + 255) / 256)
+                                                  : (numel + kFlatTileElems - 1) / kFlatTileElems;
+    if (tiles64 > (int64_t(1) << 31)) return SKEW_EINVAL;
+    const TileGeom G = plan_geometry(kind, momentum, wg_aligned, n, m, numel);
+    const bool fact = kind == kKindFactored, row = fact && G.rowpath;
+    const uint32_t nA = fact && !row ? G.ntiles : 0, nR = row ? G.rtiles : 0, nF = fact ? G.nfr + G.nfc : 0;
+    const uint32_t nB = row ? 0 : G.ntiles, nC = G.ntiles;
 
     // ---- scratch layout inside the fixed array --------------------------------------
     size_t off = 0;
     const size_t o_scal = off;   off = align256(off + sizeof(TensorScal));
+    const size_t o_fb = off;     off = align256(off + 8);
+    const size_t o_err = off;    off = align256(off + 16);
     const size_t o_tens = off;   off = align256(off + sizeof(TensorDev));
     const size_t o_iA = off;     off = align256(off + sizeof(uint2) * nA);
+    const size_t o_iR = off;     off = align256(off + sizeof(uint2) * nR);
     const size_t o_iF = off;     off = align256(off + sizeof(uint2) * nF);
-    const size_t o_iBC = off;    off = align256(off + sizeof(uint2) * nBC);
-    size_t o_rowp = 0, o_colp = 0, o_bsc = 0, o_rsum = 0;
-    if (kind == kKindFactored) {
-        o_rowp = off; off = align256(off + 4 * size_t(strips) * n);
-        o_colp = off; off = align256(off + 4 * size_t(rowtiles) * m);
+    const size_t o_iB = off;     off = align256(off + sizeof(uint2) * nB);
+    const size_t o_iC = off;     off = align256(off + sizeof(uint2) * nC);
+    size_t o_rowp = 0, o_colp = 0, o_bsc = 0, o_rsum = 0, o_pp = 0, o_rmin = 0, o_fsum = 0, o_fmin = 0;
+    if (fact && !row) {
+        o_rowp = off; off = align256(off + 4 * size_t(G.strips) * n);
+        o_colp = off; off = align256(off + 4 * size_t(G.rowtiles) * m);
         o_bsc = off;  off = align256(off + 4 * size_t(m));
-        o_rsum = off; off = align256(off + 8 * size_t(nfr));
+        o_rsum = off; off = align256(off + 8 * size_t(G.nfr));
+    } else if (row) {
+        o_colp = off; off = align256(off + 4 * size_t(G.rtiles) * m);
+        o_pp = off;   off = align256(off + 8 * size_t(G.rtiles) * m);
+        o_bsc = off;  off = align256(off + 4 * size_t(m));
+        o_rsum = off; off = align256(off + 8 * size_t(G.rtiles));
+        o_rmin = off; off = align256(off + 4 * size_t(G.rtiles));
+        o_fsum = off; off = align256(off + 8 * size_t(G.nfc));
+        o_fmin = off; off = align256(off + 4 * size_t(G.nfc));
     }
-    const size_t o_u2 = off;     off = align256(off + 8 * size_t(ntiles));
+    const size_t o_u2 = off;     off = align256(off + 8 * size_t(G.ntiles));
     if (off > SKEW_NOALLOC_SCRATCH_BYTES) return SKEW_ETOOBIG;  // too large for the fixed array
 
     // ---- device address of the fixed array, once per device ------------------------
@@ -163,10 +180,14 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     td.v = v;
     td.R = R;
     td.C = Cc;
-    td.rowp = kind == kKindFactored ? (float *)(base + o_rowp) : nullptr;
-    td.colp = kind == kKindFactored ? (float *)(base + o_colp) : nullptr;
-    td.bsc = kind == kKindFactored ? (float *)(base + o_bsc) : nullptr;
-    td.rsum = kind == kKindFactored ? (double *)(base + o_rsum) : nullptr;
+    td.rowp = fact && !row ? (float *)(base + o_rowp) : nullptr;
+    td.colp = fact ? (float *)(base + o_colp) : nullptr;
+    td.bsc = fact ? (float *)(base + o_bsc) : nullptr;
+    td.rsum = fact ? (double *)(base + o_rsum) : nullptr;
+    td.pp = row ? (double *)(base + o_pp) : nullptr;
+    td.rmin = row ? (float *)(base + o_rmin) : nullptr;
+    td.fsum = row ? (double *)(base + o_fsum) : nullptr;
+    td.fmin = row ? (float *)(base + o_fmin) : nullptr;
     td.u2 = (float2 *)(base + o_u2);
     td.n = n;
     td.m = m;
@@ -179,13 +200,17 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     bool vec = al16(td.w) && al16(td.g) && (!td.M || al16(td.M));
     vec = kind == kKindFull ? (vec && numel % 8 == 0 && al16(td.v)) : (vec && m % 8 == 0);
     td.vec = vec ? 1 : 0;
-    td.lcl = lcl;
-    td.strips = strips;
-    td.rowtiles = rowtiles;
-    td.tile_rows = tile_rows;
-    td.ntiles = ntiles;
-    td.nfr = nfr;
-    td.nfc = nfc;
+    td.lcl = G.lcl;
+    td.strips = G.strips;
+    td.rowtiles = G.rowtiles;
+    td.tile_rows = G.tile_rows;
+    td.ntiles = G.ntiles;
+    td.nfr = G.nfr;
+    td.nfc = G.nfc;
+    td.rowpath = G.rowpath;
+    td.cr = G.cr;
+    td.rt_rows = G.rt_rows;
+    td.rtiles = G.rtiles;
 
     // ---- per-step scalars, as skew_step forms them ------------------------------------
     const double t = (double)step;
@@ -194,6 +219,8 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     StepArgs a{};
     a.tensors = (const TensorDev *)(base + o_tens);
     a.scal = (TensorScal *)(base + o_scal);
+    a.err = (uint32_t *)(base + o_err);
+    a.fb = (uint32_t *)(base + o_fb);
     a.b1 = H.beta1;
     a.b2 = H.beta2;
     a.c1 = (float)(1.0 - (double)H.beta1);
@@ -208,14 +235,22 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     a.seed_lo = (uint32_t)seed;
     a.seed_hi = (uint32_t)(seed >> 32);
 
+    uint32_t nFB = 0;
+    if (row) {  // the phase-B launch a queued row-path tensor gets (as skew_bind sizes it)
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return SKEW_ECUDA;
+        nFB = (uint32_t)(2 * (sms > 0 ? sms : 1));
+    }
+
     cudaStream_t s = (cudaStream_t)stream;
+    SetupTables tb{(uint2 *)(base + o_iA), nA, (uint2 *)(base + o_iR), nR, (uint2 *)(base + o_iF), nF,
+                   (uint2 *)(base + o_iB), nB, (uint2 *)(base + o_iC), nC};
     k_noalloc_setup<<<8, 256, 0, s>>>(td, (TensorDev *)(base + o_tens), (TensorScal *)(base + o_scal),
-                                      (uint2 *)(base + o_iA), nA, (uint2 *)(base + o_iF), nF, (uint2 *)(base + o_iBC),
-                                      nBC);
+                                      (uint32_t *)(base + o_fb), tb);
     e = cudaGetLastError();
     if (e != cudaSuccess) return SKEW_ECUDA;
-    const LaunchPlan lp{nA, nF, nBC, (const uint2 *)(base + o_iA), (const uint2 *)(base + o_iF),
-                        (const uint2 *)(base + o_iBC)};
+    const LaunchPlan lp{nA, nR, nF, nB, nFB, nC, (const uint2 *)(base + o_iA), (const uint2 *)(base + o_iR),
+                        (const uint2 *)(base + o_iF), (const uint2 *)(base + o_iB), (const uint2 *)(base + o_iC)};
     e = (cudaError_t)launch_phases(a, lp, stream, nullptr);
     if (e != cudaSuccess) return SKEW_ECUDA;
     return SKEW_OK;

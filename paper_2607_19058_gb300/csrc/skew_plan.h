@@ -1,5 +1,6 @@
-// Internal layout shared by the host planner (skew_host.cpp) and the device
-// kernels (skew_kernels.cu) of libskewadam. Not part of the public ABI.
+// Internal layout shared by the host planner (skew_host.cpp), the no-alloc
+// entry point (skew_noalloc.cu) and the device kernels (skew_kernels.cu) of
+// libskewadam. Not part of the public ABI.
 #pragma once
 
 #include <stdint.h>
@@ -8,14 +9,64 @@
 namespace skew {
 
 // Every kernel runs 256-thread CTAs; a thread owns 8 consecutive bf16 elements
-// (one 16-byte vector) of up to kVecPerThread rows (factored tiles) or flat
-// vectors (full-second-moment tiles). A tile is therefore 32 Ki elements.
+// (one 16-byte vector) of up to kVecPerThread rows (strip tiles) or flat
+// vectors (full-second-moment tiles). A tile is therefore 64 Ki elements.
 constexpr int kThreads = 256;
 constexpr int kVecPerThread = 32;
 constexpr int64_t kFlatTileElems = int64_t(kThreads) * kVecPerThread * 8;
 constexpr int kFinChunk = 256;  // rows / columns per finalize item
 
+// Row-tile path (phase A on whole rows, no phase B unless a clamp may bind):
+// a chunk is kRowChunkBytes of consecutive whole rows of the bf16 gradient,
+// copied to shared memory by one bulk copy; a row tile is kRowChunks chunks;
+// the CTA keeps kRowStages chunks in flight.
+constexpr int kRowChunkBytes = 32768;
+constexpr int kRowChunks = 32;
+constexpr int kRowStages = 3;
+
 enum Kind : uint32_t { kKindFull = 0, kKindFactored = 1 };
+
+// Tile geometry of one tensor (shared by every entry point, so that the same
+// tensor is always cut the same way and results are bit-identical).
+struct TileGeom {
+    uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
+    uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0;
+};
+
+// `kind`, `momentum` as resolved by the tier policy; `wg_aligned`: weight and
+// gradient pointers are 16-byte aligned. Counts fit 32 bits for n, m <= 2^40
+// and n*m <= 2^62 only when the caller has checked the tile count (planner).
+inline TileGeom plan_geometry(uint32_t kind, uint32_t momentum, bool wg_aligned, int64_t n, int64_t m, int64_t numel) {
+    TileGeom g;
+    if (kind == kKindFactored) {
+        const int64_t vecs = (m + 7) / 8;  // 8-column groups per row
+        uint32_t lc = 1;
+        while (lc < 32 && lc < vecs) {
+            lc <<= 1;
+            ++g.lcl;
+        }
+        g.strips = (uint32_t)((m + 8 * lc - 1) / (8 * lc));
+        g.tile_rows = (uint32_t)(kVecPerThread * (kThreads / lc));
+        g.rowtiles = (uint32_t)((n + g.tile_rows - 1) / g.tile_rows);
+        g.ntiles = g.strips * g.rowtiles;
+        g.nfc = (uint32_t)((m + kFinChunk - 1) / kFinChunk);
+        // Whole-row phase A: momentum-free factored matrices of width 2048 or
+        // 4096 (one or two 16-byte vectors per thread per row).
+        g.rowpath = (!momentum && wg_aligned && (m == 2048 || m == 4096)) ? 1u : 0u;
+        if (g.rowpath) {
+            g.cr = (uint32_t)(kRowChunkBytes / (2 * m));
+            g.rt_rows = g.cr * kRowChunks;
+            g.rtiles = (uint32_t)((n + g.rt_rows - 1) / g.rt_rows);
+            g.nfr = 0;
+        } else {
+            g.nfr = (uint32_t)((n + kFinChunk - 1) / kFinChunk);
+        }
+    } else {
+        g.rowtiles = (uint32_t)((numel + kFlatTileElems - 1) / kFlatTileElems);
+        g.ntiles = g.rowtiles;
+    }
+    return g;
+}
 
 // Device descriptor of one tensor (lives in the workspace).
 struct TensorDev {
@@ -25,10 +76,14 @@ struct TensorDev {
     float *v;           // exact second moment (numel) or null
     float *R;           // row factor (n) or null
     float *C;           // column factor (m) or null
-    float *rowp;        // factored: row partials [strips][n]
-    float *colp;        // factored: column partials [rowtiles][m]
+    float *rowp;        // strip path: row partials [strips][n]
+    float *colp;        // factored: column partials of g^2 [rowtiles or rtiles][m]
     float *bsc;         // factored: 1/sqrt(C_j) [m]
-    double *rsum;       // factored: per finalize-row-item sum of R [nfr]
+    double *rsum;       // factored: sums of R per finalize-row item [nfr] / per row tile [rtiles]
+    double *pp;         // row path: column partials of g^2 / R_i [rtiles][m]
+    float *rmin;        // row path: smallest positive R_i per row tile [rtiles]
+    double *fsum;       // row path: sum of P_j / C_j per finalize item [nfc]
+    float *fmin;        // row path: smallest C_j with P_j > 0 per finalize item [nfc]
     float2 *u2;         // per tile sum of (U / coef)^2 as a (hi, lo) pair [ntiles]
     int64_t n, m, numel;
     uint32_t tid;       // dither tensor id
@@ -37,23 +92,29 @@ struct TensorDev {
     uint32_t lcl;       // factored: log2 of lanes along a row (LC)
     uint32_t strips;    // factored: column strips of 8*LC columns
     uint32_t rowtiles;  // factored: row tiles of tile_rows rows; full: flat tiles
-    uint32_t tile_rows; // factored: rows per tile = 16 * (256 / LC)
+    uint32_t tile_rows; // factored: rows per tile = 32 * (256 / LC)
     uint32_t ntiles;    // update tiles of this tensor
     uint32_t nfr, nfc;  // factored: finalize items over rows / columns
+    uint32_t rowpath;   // 1: whole-row phase A (k_rowsq) and the bilinear sum of U^2
+    uint32_t cr;        // row path: rows per chunk
+    uint32_t rt_rows;   // row path: rows per row tile
+    uint32_t rtiles;    // row path: row tiles
 };
 
 // Per-tensor scalars of the current step (zeroed at the start of every step).
 struct TensorScal {
-    double rbar;      // mean(R)
-    double sumsq;     // sum over the tensor of U^2
-    double rms;       // RMS(U)
-    double kappa;     // 1 / max(1, RMS / d)
-    float rbar_s;     // mean(R) * 2^rbar_e, in [1, 2); 0 if mean(R) == 0
+    double rbar;        // mean(R)
+    double sumsq;       // sum over the tensor of U^2
+    double rms;         // RMS(U)
+    double kappa;       // 1 / max(1, RMS / d)
+    float rbar_s;       // mean(R) * 2^rbar_e, in [1, 2); 0 if mean(R) == 0
     int32_t rbar_e;
-    float coefC;      // lr * kappa * coef, the factor applied to (y / D)
-    uint32_t cntF;    // finalize items done
-    uint32_t cntB;    // update-RMS tiles done
-    uint32_t pad[3];
+    float coefC;        // lr * kappa * coef, the factor applied to (y / D)
+    uint32_t cntF;      // finalize items done
+    uint32_t cntB;      // update-RMS tiles done
+    uint32_t fallback;  // row path: 1 if sum(U^2) needs phase B (a clamp may bind)
+    uint32_t zflag;     // row path: a row with R_i == 0 holds a nonzero gradient
+    uint32_t pad;
 };
 static_assert(sizeof(TensorScal) == 64, "TensorScal layout");
 
@@ -61,6 +122,8 @@ static_assert(sizeof(TensorScal) == 64, "TensorScal layout");
 struct StepArgs {
     const TensorDev *tensors;
     TensorScal *scal;
+    uint32_t *err;         // sticky status word (nonzero: a bounded wait gave up)
+    uint32_t *fb;          // [0]: row-path tensors that need phase B, [1..]: their ids
     float b1, b2, c1, c2;  // beta1, beta2, 1-beta1, 1-beta2 (fp32)
     float ce;              // 1 / sqrt(eps), fp32
     float wdf;             // 1 - lr * lambda, fp32
@@ -72,17 +135,25 @@ struct StepArgs {
     uint32_t seed_lo, seed_hi;
 };
 
-// The four phases of a set of tensors: item lists (tensor, local tile / item)
-// in device memory and their lengths.
+// The phases of one step: item lists (tensor, local tile / item) in device
+// memory and their lengths.
+//   A  strip-tile sums of squares (strip-path factored tensors)
+//   R  row-tile sums of squares and bilinear partials (row-path tensors)
+//   F  finalize items (rows and columns; columns only on the row path)
+//   B  update-RMS tiles (strip-path factored and full tensors)
+//   FB phase B of the row-path tensors whose finalize asked for it (nFB CTAs)
+//   C  apply tiles (every tensor)
 struct LaunchPlan {
-    uint32_t nA, nF, nBC;
-    const uint2 *itemsA, *itemsF, *itemsBC;
+    uint32_t nA, nR, nF, nB, nFB, nC;
+    const uint2 *itemsA, *itemsR, *itemsF, *itemsB, *itemsC;
 };
 
-// Enqueues the phases of `L` as four grouped launches (A, F, B, C) on `stream`,
-// each given the step parameters A by value. If `ev` is not null it holds five
-// cudaEvent_t, recorded before the first launch and after each of the four.
-// Returns a cudaError_t value.
+constexpr int kLaunches = 6;
+
+// Enqueues the phases of `L` as grouped launches (A, R, F, B, FB, C; empty ones
+// skipped) on `stream`, each given the step parameters by value. If `ev` is not
+// null it holds kLaunches + 1 cudaEvent_t, recorded before the first launch and
+// after each of the six. Returns a cudaError_t value.
 int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *const *ev);
 
 }  // namespace skew

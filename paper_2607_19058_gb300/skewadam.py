@@ -50,7 +50,8 @@ class HParams(C.Structure):
 class TensorInfo(C.Structure):
     _fields_ = [("kind", C.c_int32), ("momentum", C.c_int32), ("decay", C.c_int32), ("vectorized", C.c_int32),
                 ("rows", C.c_int64), ("cols", C.c_int64), ("numel", C.c_int64), ("m_offset", C.c_int64),
-                ("v_offset", C.c_int64), ("r_offset", C.c_int64), ("c_offset", C.c_int64)]
+                ("v_offset", C.c_int64), ("r_offset", C.c_int64), ("c_offset", C.c_int64), ("rowpath", C.c_int32),
+                ("reserved", C.c_int32)]
 
 
 _lock = threading.Lock()

@@ -195,3 +195,31 @@ def test_ablation_awkward_full_size_subset():
     for t in (1, 2):
         h.step(t)
     h.close()
+
+
+def _row_path_workload():
+    """Momentum-free matrices of width 4096 / 2048 (the whole-row phase A): ragged
+    row tiles and chunks, and expert 5 with zero gradients on odd steps."""
+    E = WL.TIER_EXPERT
+    specs = [WL.Spec("e512x4096", (512, 4096), E, expert=0), WL.Spec("e301x4096", (301, 4096), E, expert=1),
+             WL.Spec("e1000x2048", (1000, 2048), E, expert=2), WL.Spec("e77x2048", (77, 2048), E, expert=3),
+             WL.Spec("zero_odd", (256, 4096), E, expert=5)]
+    return WL.Workload("rowpath", specs, WL.HP(), "toy", steps=4)
+
+
+def test_row_path_bilinear_sum():
+    """eps = 1e-30: no clamp can bind, so sum(U^2) comes from the whole-row partials."""
+    h = _harness(_row_path_workload())
+    assert all(h.opt.info(k).rowpath == 1 for k in range(len(h.wl.specs)))
+    for t in range(1, 5):
+        h.step(t, seed=t * 31)
+    h.close()
+
+
+def test_row_path_clamp_falls_back_to_phase_b():
+    """eps = 1e-8 (App. A): the clamp binds at step 1, so the finalize queues the
+    tensors for phase B and sum(U^2) is taken element by element."""
+    h = _harness(_row_path_workload(), hp_override=dict(eps=1e-8, lr=3e-4, weight_decay=0.05))
+    for t in range(1, 4):
+        h.step(t, seed=77)
+    h.close()

@@ -20,8 +20,10 @@ from paper_2607_19058_gb300 import workloads as WL
 
 pytestmark = pytest.mark.gpu
 
+# (8192, 4096) expert: a momentum-free matrix on the whole-row path; (50304, 4096)
+# backbone: the paper's embedding, the largest tensor the fixed scratch is sized for.
 SHAPES = [((300, 1000), S.TIER_EXPERT), ((517, 136), S.TIER_BACKBONE), ((4096, 127), S.TIER_ROUTER),
-          ((100003,), S.TIER_BACKBONE), ((50304, 4096), S.TIER_EXPERT)]
+          ((100003,), S.TIER_BACKBONE), ((8192, 4096), S.TIER_EXPERT), ((50304, 4096), S.TIER_BACKBONE)]
 
 
 @pytest.fixture(scope="module", autouse=True)
