@@ -27,6 +27,7 @@ scaling is weak.
 the host cores instead, on bounded samples of the same workload.
 """
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -147,6 +148,28 @@ def byte_model(opt, n_tensors):
         "k_apply": 4 * N + 2 * N_nomom + 4 * N_mom + 4 * N_full,  # W r/w; G or M; v read
     }
     return dict(N=N, N_mom=N_mom, N_full=N_full, rc=rc, step_min=step_min, kernels=kernels)
+
+
+def recorded_traffic(kernel, workload):
+    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu summary
+    (profiles/dram_traffic_appb.md, `traffic:` lines), or None when there is none or the
+    kernel source has changed since the counters were taken (its SHA-256 differs)."""
+    root = os.path.dirname(os.path.abspath(__file__))
+    src = os.path.join(root, "paper_2607_19058_gb300", "csrc", "skew_kernels.cu")
+    summ = os.path.join(root, "profiles", "dram_traffic_appb.md")
+    try:
+        with open(src, "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()
+        lines = open(summ).read().splitlines()
+    except OSError:
+        return None
+    for ln in lines:
+        if not ln.startswith("traffic:"):
+            continue
+        kv = dict(x.split("=", 1) for x in ln[len("traffic:"):].split())
+        if kv.get("kernel") == kernel and kv.get("workload") == workload and kv.get("source_sha256") == sha:
+            return int(kv["per_launch"])
+    return None
 
 
 # ---------------------------------------------------------------------------
@@ -379,7 +402,7 @@ def run_ours(args):
                     "frac_of_8tbs": step_gbs / NOMINAL_HBM_GBS, "frac_of_measured": step_gbs / peak,
                     "peak_gbs": peak, "peak_source": peak_src},
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None, "algorithmic_bytes_per_launch": dom_bytes,
+                         "frac": achieved / peak, "traffic": recorded_traffic(dom, args.workload), "algorithmic_bytes_per_launch": dom_bytes,
                          "launch_ms": kmean[dom], "peak_source": peak_src},
             "kernels_ms": kmean,
             "e2e": e2e,

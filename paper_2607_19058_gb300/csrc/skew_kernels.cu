@@ -84,6 +84,15 @@ __device__ __forceinline__ void unpack_bf8(uint4 u, float (&o)[8]) {
     }
 }
 
+// The same eight values as four (even, odd) pairs for the packed FP32x2 unit.
+__device__ __forceinline__ void unpack_bf8x2(uint4 u, float2 (&o)[4]) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) o[q] = make_float2(__uint_as_float(w[q] << 16), __uint_as_float(w[q] & 0xFFFF0000u));
+}
+
+__device__ __forceinline__ float2 neg2(float2 a) { return make_float2(-a.x, -a.y); }
+
 // Eight bf16 values (scalar path: elements >= valid read as 0).
 __device__ __forceinline__ void load_bf8_scalar(const uint16_t *p, int valid, float (&o)[8]) {
 #pragma unroll
@@ -195,6 +204,13 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     s = a + b;
     const float bp = s - a;
     e = (a - (s - bp)) + (b - bp);
+}
+
+// TwoSum on both lanes of a pair (packed FP32x2 adds; same results as two_sum).
+__device__ __forceinline__ void two_sum2(float2 a, float2 b, float2 &s, float2 &e) {
+    s = __fadd2_rn(a, b);
+    const float2 bp = __fadd2_rn(s, neg2(a));
+    e = __fadd2_rn(__fadd2_rn(a, neg2(__fadd2_rn(s, neg2(bp)))), __fadd2_rn(b, neg2(bp)));
 }
 
 // Compensated accumulator: the running sum is hi + lo.
@@ -609,11 +625,12 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const float b2 = A.b2, c2 = A.c2, fm = (float)T.m;
-    float cs[NV][8], ph[NV][8], pl[NV][8];
+    // per column pair: sums of g^2 and the compensated (hi, lo) sum of g^2 / R_i
+    float2 cs[NV][4], ph[NV][4], pl[NV][4];
 #pragma unroll
     for (int v = 0; v < NV; ++v)
 #pragma unroll
-        for (int c = 0; c < 8; ++c) cs[v][c] = ph[v][c] = pl[v][c] = 0.f;
+        for (int q = 0; q < 4; ++q) cs[v][q] = ph[v][q] = pl[v][q] = make_float2(0.f, 0.f);
     double rsum = 0.0;                       // threads < CR: sum of this lane's rows' R
     float rmin = __int_as_float(0x7F800000);  // threads < CR: smallest positive R of this lane's rows
     bool zero_row = false;
@@ -631,20 +648,21 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         float rs[CR];
 #pragma unroll
         for (int r = 0; r < CR; ++r) {
-            rs[r] = 0.f;
+            float2 r2 = make_float2(0.f, 0.f);
             if (r < (int)ch.rows) {
 #pragma unroll
                 for (int v = 0; v < NV; ++v) {
-                    float g[8];
-                    unpack_bf8(buf[r * V + v * kThreads + tid], g);
+                    float2 g[4];
+                    unpack_bf8x2(buf[r * V + v * kThreads + tid], g);
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        const float q = g[k] * g[k];
-                        cs[v][k] += q;
-                        rs[r] += q;
+                    for (int q = 0; q < 4; ++q) {
+                        const float2 sq = __fmul2_rn(g[q], g[q]);
+                        cs[v][q] = __fadd2_rn(cs[v][q], sq);
+                        r2 = __fadd2_rn(r2, sq);
                     }
                 }
             }
+            rs[r] = r2.x + r2.y;
         }
         int j;
         const float tot = warp_sum_transposed<CR>(rs, j);
@@ -674,32 +692,33 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         }
         __syncthreads();
         // pass 2: P_j += g^2 / R_i, a chunk sum per column folded into (hi, lo)
-        float t[NV][8];
+        float2 t[NV][4];
 #pragma unroll
         for (int v = 0; v < NV; ++v)
 #pragma unroll
-            for (int k = 0; k < 8; ++k) t[v][k] = 0.f;
+            for (int q = 0; q < 4; ++q) t[v][q] = make_float2(0.f, 0.f);
 #pragma unroll
         for (int r = 0; r < CR; ++r) {
             if (r < (int)ch.rows) {
                 const float iv = sm.inv[r];
+                const float2 iv2 = make_float2(iv, iv);
 #pragma unroll
                 for (int v = 0; v < NV; ++v) {
-                    float g[8];
-                    unpack_bf8(buf[r * V + v * kThreads + tid], g);
+                    float2 g[4];
+                    unpack_bf8x2(buf[r * V + v * kThreads + tid], g);
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) t[v][k] = fmaf(g[k] * g[k], iv, t[v][k]);
+                    for (int q = 0; q < 4; ++q) t[v][q] = __ffma2_rn(__fmul2_rn(g[q], g[q]), iv2, t[v][q]);
                 }
             }
         }
 #pragma unroll
         for (int v = 0; v < NV; ++v)
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                float s2, e;
-                two_sum(ph[v][k], t[v][k], s2, e);
-                ph[v][k] = s2;
-                pl[v][k] += e;
+            for (int q = 0; q < 4; ++q) {
+                float2 s2, e2;
+                two_sum2(ph[v][q], t[v][q], s2, e2);
+                ph[v][q] = s2;
+                pl[v][q] = __fadd2_rn(pl[v][q], e2);
             }
     }
     if (c < nch) {
@@ -721,13 +740,12 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
     for (int v = 0; v < NV; ++v) {
         const int64_t col = 8 * int64_t(v * kThreads + tid);
         float4 *cp4 = reinterpret_cast<float4 *>(T.colp + base + col);
-        cp4[0] = make_float4(cs[v][0], cs[v][1], cs[v][2], cs[v][3]);
-        cp4[1] = make_float4(cs[v][4], cs[v][5], cs[v][6], cs[v][7]);
+        cp4[0] = make_float4(cs[v][0].x, cs[v][0].y, cs[v][1].x, cs[v][1].y);
+        cp4[1] = make_float4(cs[v][2].x, cs[v][2].y, cs[v][3].x, cs[v][3].y);
         double2 *pp2 = reinterpret_cast<double2 *>(T.pp + base + col);
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-            pp2[k] = make_double2((double)ph[v][2 * k] + (double)pl[v][2 * k],
-                                  (double)ph[v][2 * k + 1] + (double)pl[v][2 * k + 1]);
+        for (int q = 0; q < 4; ++q)
+            pp2[q] = make_double2((double)ph[v][q].x + (double)pl[v][q].x, (double)ph[v][q].y + (double)pl[v][q].y);
     }
     if (zero_row) atomicOr(&S.zflag, 1u);
     if (warp == 0) {
@@ -1124,8 +1142,15 @@ __device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const Ten
                     const float a = rows[(k0 + q) * RG];
                     if constexpr (FAST) {
                         const float ca = -coefC * a;
+                        const float2 ca2 = make_float2(ca, ca), wdf2 = make_float2(wdf, wdf);
 #pragma unroll
-                        for (int c = 0; c < 8; ++c) x[c] = fmaf(ca * b[c], y[c], w[c] * wdf);
+                        for (int q = 0; q < 4; ++q) {
+                            const float2 xx = __ffma2_rn(__fmul2_rn(ca2, make_float2(b[2 * q], b[2 * q + 1])),
+                                                         make_float2(y[2 * q], y[2 * q + 1]),
+                                                         __fmul2_rn(make_float2(w[2 * q], w[2 * q + 1]), wdf2));
+                            x[2 * q] = xx.x;
+                            x[2 * q + 1] = xx.y;
+                        }
                     } else {
 #pragma unroll
                         for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], ce), w[c] * wdf);
