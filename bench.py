@@ -145,7 +145,8 @@ def byte_model(opt, n_tensors):
         "k_finalize": 8 * (rc + rc_row),                         # R, C read + write
         "k_rms": 2 * (N - N_row) + 8 * N_mom + 8 * N_full,       # read G; M, v read + write
         "k_fallback": 0,                                          # runs only when a clamp may bind
-        "k_apply": 4 * N + 2 * N_nomom + 4 * N_mom + 4 * N_full,  # W r/w; G or M; v read
+        "k_apply": 4 * (N - N_row) + 2 * (N_nomom - N_row) + 4 * N_mom + 4 * N_full,  # W r/w; G or M; v read
+        "k_apply_rows": 6 * N_row,                               # row path: W r/w, G read
     }
     return dict(N=N, N_mom=N_mom, N_full=N_full, rc=rc, step_min=step_min, kernels=kernels)
 

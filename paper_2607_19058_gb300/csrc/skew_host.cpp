@@ -46,8 +46,8 @@ struct skew_handle {
     std::vector<TPlan> t;
     size_t state_bytes = 0, ws_bytes = 0;
     size_t ws_scal = 0, ws_fb = 0, ws_err = 0, ws_tab = 0, ws_tab_end = 0;
-    size_t ws_tens = 0, ws_itemsA = 0, ws_itemsR = 0, ws_itemsF = 0, ws_itemsB = 0, ws_itemsC = 0;
-    std::vector<uint2> itemsA, itemsR, itemsF, itemsB, itemsC;  // per phase, tensors in order
+    size_t ws_tens = 0, ws_itemsA = 0, ws_itemsR = 0, ws_itemsF = 0, ws_itemsB = 0, ws_itemsC = 0, ws_itemsCR = 0;
+    std::vector<uint2> itemsA, itemsR, itemsF, itemsB, itemsC, itemsCR;  // per phase, tensors in order
     uint32_t n_rowpath = 0;  // tensors on the row path
     uint32_t fb_ctas = 0;    // CTAs of the row path's phase-B launch (set at bind)
     char *state = nullptr, *ws = nullptr;
@@ -63,7 +63,8 @@ struct skew_handle {
 
 // What the profiler times per step: the grouped launches (an empty phase times ~0).
 constexpr int kProfLaunches = kLaunches;
-const char *const kProfNames[kProfLaunches] = {"k_sumsq", "k_rowsq", "k_finalize", "k_rms", "k_fallback", "k_apply"};
+const char *const kProfNames[kProfLaunches] = {"k_sumsq", "k_rowsq",  "k_finalize", "k_rms",
+                                               "k_fallback", "k_apply", "k_apply_rows"};
 
 static int fail(skew_handle_t *h, int code, const char *fmt, ...) {
     char buf[512];
@@ -195,9 +196,12 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
                     for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsA.push_back(make_uint2(q, i));
                 for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(q, i));
             }
-            if (!p.rowpath)
+            if (p.rowpath) {
+                for (uint32_t i = 0; i < p.rtiles; ++i) h->itemsCR.push_back(make_uint2(q, i));
+            } else {
                 for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsB.push_back(make_uint2(q, i));
-            for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsC.push_back(make_uint2(q, i));
+                for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsC.push_back(make_uint2(q, i));
+            }
         }
     } catch (...) {
         delete h;
@@ -225,6 +229,7 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     table(h->ws_itemsF, h->itemsF);
     table(h->ws_itemsB, h->itemsB);
     table(h->ws_itemsC, h->itemsC);
+    table(h->ws_itemsCR, h->itemsCR);
     h->ws_tab_end = w;
     for (auto &p : h->t) {
         if (p.kind == kKindFactored && !p.rowpath) {
@@ -263,7 +268,8 @@ int32_t skew_num_tensors(const skew_handle_t *h) { return h ? (int32_t)h->t.size
 int64_t skew_launches_per_step(const skew_handle_t *h) {
     if (!h) return 0;
     return int64_t(!h->itemsA.empty()) + int64_t(!h->itemsR.empty()) + int64_t(!h->itemsF.empty()) +
-           int64_t(!h->itemsB.empty()) + int64_t(h->n_rowpath > 0) + int64_t(!h->itemsC.empty());
+           int64_t(!h->itemsB.empty()) + int64_t(h->n_rowpath > 0) + int64_t(!h->itemsC.empty()) +
+           int64_t(!h->itemsCR.empty());
 }
 
 const char *skew_last_error(const skew_handle_t *h) { return h ? h->err.c_str() : g_create_err.c_str(); }
@@ -363,6 +369,7 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
     put(h->ws_itemsF, h->itemsF);
     put(h->ws_itemsB, h->itemsB);
     put(h->ws_itemsC, h->itemsC);
+    put(h->ws_itemsCR, h->itemsCR);
 
     cudaError_t e;
     if (!img.empty()) {
@@ -433,8 +440,8 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
     auto items = [&](size_t at) { return reinterpret_cast<const uint2 *>(h->ws + at); };
     const LaunchPlan L{(uint32_t)h->itemsA.size(), (uint32_t)h->itemsR.size(), (uint32_t)h->itemsF.size(),
                        (uint32_t)h->itemsB.size(), h->n_rowpath ? h->fb_ctas : 0u, (uint32_t)h->itemsC.size(),
-                       items(h->ws_itemsA), items(h->ws_itemsR), items(h->ws_itemsF), items(h->ws_itemsB),
-                       items(h->ws_itemsC)};
+                       (uint32_t)h->itemsCR.size(), items(h->ws_itemsA), items(h->ws_itemsR), items(h->ws_itemsF),
+                       items(h->ws_itemsB), items(h->ws_itemsC), items(h->ws_itemsCR)};
     e = (cudaError_t)launch_phases(a, L, s, reinterpret_cast<void *const *>(ev));
     if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
     return SKEW_OK;

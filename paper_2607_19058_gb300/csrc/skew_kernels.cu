@@ -1206,6 +1206,157 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
 }
 
 // ---------------------------------------------------------------------------
+// Row path, phase C (k_apply_rows): the row tiles of k_rowsq. A chunk is CA
+// whole rows of W and the same rows of G, one bulk copy each into a ring slot
+// (W in the first half, G in the second); the column scales b_j of a thread's
+// 8*NV columns stay in registers and the tile's row scales a_i in shared memory.
+// Per element the arithmetic, the dither index and the rounding are those of
+// apply_fact_tile, so the result is the same bit for bit.
+// ---------------------------------------------------------------------------
+struct ApplyRowSmem {
+    uint4 buf[kRowStages][kRowChunkBytes / 16];  // [W rows | G rows] per slot
+    uint64_t full[kRowStages];
+    float a[kRowChunks * 8];                     // row scales a_i of the tile (rt_rows <= 256)
+    float red[2 * kThreads / 32];
+};
+
+__device__ __forceinline__ void apply_row_issue(const TensorDev &T, uint32_t tile, uint32_t c, uint32_t ca,
+                                                ApplyRowSmem &sm, uint64_t pol) {
+    const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * ca;
+    const uint32_t rows = (uint32_t)min((int64_t)ca, T.n - i0);
+    const uint32_t bytes = rows * (uint32_t)T.m * 2u;
+    const int st = c % kRowStages;
+    mbar_expect_tx(&sm.full[st], 2u * bytes);
+    bulk_g2s(sm.buf[st], T.w + i0 * T.m, bytes, &sm.full[st], pol);
+    bulk_g2s(sm.buf[st] + kRowChunkBytes / 32, T.g + i0 * T.m, bytes, &sm.full[st], pol);
+}
+
+template <int NV, bool FAST>
+__device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t tile, const float (&b)[NV][8],
+                                float coefC, ApplyRowSmem &sm, uint32_t nch, uint32_t ca, uint64_t pol) {
+    constexpr int V = kThreads * NV;       // vectors per row
+    constexpr int CA = 4 / NV;             // rows per chunk (16 KB of W, 16 KB of G)
+    const int tid = threadIdx.x;
+    const int64_t m = T.m;
+    uint16_t *__restrict__ w_ = T.w;
+    const Dith d = dith_of(A, T.tid);
+    const float wdf = T.decay ? A.wdf : 1.0f;
+    const float ce = A.ce;
+    const float2 wdf2 = make_float2(wdf, wdf);
+    const Pol sp;
+    for (uint32_t c = 0; c < nch; ++c) {
+        const int st = c % kRowStages;
+        const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * ca;
+        const int rows = (int)min((int64_t)CA, T.n - i0);
+        const bool ok = mbar_wait(&sm.full[st], (c / kRowStages) & 1u);
+        const uint4 *bw = sm.buf[st];
+        const uint4 *bg = sm.buf[st] + kRowChunkBytes / 32;
+#pragma unroll
+        for (int r = 0; r < CA; ++r) {
+            if (r < rows) {
+                const float a = sm.a[c * CA + r];
+                const float cr = -coefC * a;
+                const float2 cr2 = make_float2(cr, cr);
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    float y[8], w[8], x[8];
+                    unpack_bf8(bg[r * V + v * kThreads + tid], y);
+                    unpack_bf8(bw[r * V + v * kThreads + tid], w);
+                    if constexpr (FAST) {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const float2 xx =
+                                __ffma2_rn(__fmul2_rn(cr2, make_float2(b[v][2 * q], b[v][2 * q + 1])),
+                                           make_float2(y[2 * q], y[2 * q + 1]),
+                                           __fmul2_rn(make_float2(w[2 * q], w[2 * q + 1]), wdf2));
+                            x[2 * q] = xx.x;
+                            x[2 * q + 1] = xx.y;
+                        }
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) x[k] = fmaf(-coefC, y[k] * fminf(a * b[v][k], ce), w[k] * wdf);
+                    }
+                    write8<true>(w_, d, (i0 + r) * m + 8 * (v * kThreads + tid), 8, true, x, sp);
+                }
+            }
+        }
+        // every thread is done with slot st: refill it with chunk c + kRowStages
+        if (__syncthreads_or(!ok)) {
+            if (tid == 0) {
+                atomicOr(A.err, 2u);
+                const uint32_t issued_end = min(nch, c + kRowStages);  // chunks [0, c + kRowStages) were issued
+                for (uint32_t k = c; k < issued_end; ++k)
+                    (void)mbar_wait(&sm.full[k % kRowStages], (k / kRowStages) & 1u);
+            }
+            return;
+        }
+        if (tid == 0 && c + kRowStages < nch) {
+            fence_proxy_async_smem();
+            apply_row_issue(T, tile, c + kRowStages, ca, sm, pol);
+        }
+    }
+}
+
+template <int NV>
+__device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile,
+                                ApplyRowSmem &sm) {
+    constexpr int CA = 4 / NV;
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    const int64_t r0 = int64_t(tile) * T.rt_rows;
+    const uint32_t rows_t = (uint32_t)min((int64_t)T.rt_rows, T.n - r0);
+    const uint32_t nch = (rows_t + CA - 1) / CA;
+    if (threadIdx.x == 0) {
+        for (int st = 0; st < kRowStages; ++st) mbar_init(&sm.full[st], 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+        for (uint32_t c = 0; c < nch && c < (uint32_t)kRowStages; ++c) apply_row_issue(T, tile, c, CA, sm, pol);
+    // row scales of the tile, column scales of this thread's columns, and the clamp test
+    const float rbar_s = __ldcg(&S.rbar_s);
+    const int rbar_e = __ldcg(&S.rbar_e);
+    float ma = 0.f, mb = 0.f;
+    for (uint32_t r = threadIdx.x; r < rows_t; r += kThreads) {
+        const float a = row_scale(__ldcg(T.R + r0 + r), rbar_s, rbar_e);
+        sm.a[r] = a;
+        ma = fmaxf(ma, nan_to_inf(a));
+    }
+    float b[NV][8];
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+        const float *p = T.bsc + 8 * (v * kThreads + threadIdx.x);
+        const float4 b0 = __ldcg(reinterpret_cast<const float4 *>(p));
+        const float4 b1 = __ldcg(reinterpret_cast<const float4 *>(p + 4));
+        b[v][0] = b0.x; b[v][1] = b0.y; b[v][2] = b0.z; b[v][3] = b0.w;
+        b[v][4] = b1.x; b[v][5] = b1.y; b[v][6] = b1.z; b[v][7] = b1.w;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mb = fmaxf(mb, nan_to_inf(b[v][k]));
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        ma = fmaxf(ma, __shfl_xor_sync(kAll, ma, o));
+        mb = fmaxf(mb, __shfl_xor_sync(kAll, mb, o));
+    }
+    if ((threadIdx.x & 31) == 0) {
+        sm.red[threadIdx.x >> 5] = ma;
+        sm.red[kThreads / 32 + (threadIdx.x >> 5)] = mb;
+    }
+    __syncthreads();
+    ma = mb = 0.f;
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w) {
+        ma = fmaxf(ma, sm.red[w]);
+        mb = fmaxf(mb, sm.red[kThreads / 32 + w]);
+    }
+    const float coefC = __ldcg(&S.coefC);
+    if (ma * mb <= A.ce)
+        apply_rows_body<NV, true>(A, T, tile, b, coefC, sm, nch, CA, pol);
+    else
+        apply_rows_body<NV, false>(A, T, tile, b, coefC, sm, nch, CA, pol);
+}
+
+// ---------------------------------------------------------------------------
 // Kernels: one tile / item per CTA. The per-step parameters are a kernel
 // parameter (constant bank), so the dither keys and step scalars are uniform
 // operands of every warp.
@@ -1232,6 +1383,19 @@ __global__ void __launch_bounds__(kThreads, 2) k_rowsq(const __grid_constant__ S
         rowsq_tile<2>(A, T, A.scal[it.x], it.y, sm);
     else
         rowsq_tile<1>(A, T, A.scal[it.x], it.y, sm);
+}
+
+// Row path, phase C: one row tile per CTA (dynamic shared memory: ApplyRowSmem).
+__global__ void __launch_bounds__(kThreads, 2)
+    k_apply_rows(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
+    extern __shared__ uint4 dyn_smem[];
+    ApplyRowSmem &sm = *reinterpret_cast<ApplyRowSmem *>(dyn_smem);
+    const uint2 it = items[blockIdx.x];
+    const TensorDev &T = A.tensors[it.x];
+    if (T.m == 4096)
+        apply_rows_tile<2>(A, T, A.scal[it.x], it.y, sm);
+    else
+        apply_rows_tile<1>(A, T, A.scal[it.x], it.y, sm);
 }
 
 // Phase B of the row-path tensors whose finalize found that a clamp may bind
@@ -1328,6 +1492,13 @@ int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *co
     mark(5);
     if (L.nC) k_apply<<<L.nC, kThreads, 0, s>>>(A, L.itemsC);
     mark(6);
+    if (L.nCR) {
+        const cudaError_t e =
+            cudaFuncSetAttribute(k_apply_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(ApplyRowSmem));
+        if (e != cudaSuccess) return (int)e;
+        k_apply_rows<<<L.nCR, kThreads, sizeof(ApplyRowSmem), s>>>(A, L.itemsCR);
+    }
+    mark(7);
     return (int)cudaGetLastError();
 }
 

@@ -44,6 +44,8 @@ struct SetupTables {
     uint32_t nB;
     uint2 *C;
     uint32_t nC;
+    uint2 *CR;
+    uint32_t nCR;
 };
 
 // Writes the descriptor, clears the scalars and the phase-B queue (the step's
@@ -61,6 +63,7 @@ __global__ void k_noalloc_setup(TensorDev td, TensorDev *dst, TensorScal *scal, 
     for (uint32_t i = i0; i < tb.nF; i += stride) tb.F[i] = make_uint2(0, i);
     for (uint32_t i = i0; i < tb.nB; i += stride) tb.B[i] = make_uint2(0, i);
     for (uint32_t i = i0; i < tb.nC; i += stride) tb.C[i] = make_uint2(0, i);
+    for (uint32_t i = i0; i < tb.nCR; i += stride) tb.CR[i] = make_uint2(0, i);
 }
 
 }  // namespace
@@ -125,7 +128,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     const TileGeom G = plan_geometry(kind, momentum, wg_aligned, n, m, numel);
     const bool fact = kind == kKindFactored, row = fact && G.rowpath;
     const uint32_t nA = fact && !row ? G.ntiles : 0, nR = row ? G.rtiles : 0, nF = fact ? G.nfr + G.nfc : 0;
-    const uint32_t nB = row ? 0 : G.ntiles, nC = G.ntiles;
+    const uint32_t nB = row ? 0 : G.ntiles, nC = row ? 0 : G.ntiles, nCR = row ? G.rtiles : 0;
 
     // ---- scratch layout inside the fixed array --------------------------------------
     size_t off = 0;
@@ -138,6 +141,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     const size_t o_iF = off;     off = align256(off + sizeof(uint2) * nF);
     const size_t o_iB = off;     off = align256(off + sizeof(uint2) * nB);
     const size_t o_iC = off;     off = align256(off + sizeof(uint2) * nC);
+    const size_t o_iCR = off;    off = align256(off + sizeof(uint2) * nCR);
     size_t o_rowp = 0, o_colp = 0, o_bsc = 0, o_rsum = 0, o_pp = 0, o_rmin = 0, o_fsum = 0, o_fmin = 0;
     if (fact && !row) {
         o_rowp = off; off = align256(off + 4 * size_t(G.strips) * n);
@@ -244,13 +248,24 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
 
     cudaStream_t s = (cudaStream_t)stream;
     SetupTables tb{(uint2 *)(base + o_iA), nA, (uint2 *)(base + o_iR), nR, (uint2 *)(base + o_iF), nF,
-                   (uint2 *)(base + o_iB), nB, (uint2 *)(base + o_iC), nC};
+                   (uint2 *)(base + o_iB), nB, (uint2 *)(base + o_iC), nC, (uint2 *)(base + o_iCR), nCR};
     k_noalloc_setup<<<8, 256, 0, s>>>(td, (TensorDev *)(base + o_tens), (TensorScal *)(base + o_scal),
                                       (uint32_t *)(base + o_fb), tb);
     e = cudaGetLastError();
     if (e != cudaSuccess) return SKEW_ECUDA;
-    const LaunchPlan lp{nA, nR, nF, nB, nFB, nC, (const uint2 *)(base + o_iA), (const uint2 *)(base + o_iR),
-                        (const uint2 *)(base + o_iF), (const uint2 *)(base + o_iB), (const uint2 *)(base + o_iC)};
+    const LaunchPlan lp{nA,
+                        nR,
+                        nF,
+                        nB,
+                        nFB,
+                        nC,
+                        nCR,
+                        (const uint2 *)(base + o_iA),
+                        (const uint2 *)(base + o_iR),
+                        (const uint2 *)(base + o_iF),
+                        (const uint2 *)(base + o_iB),
+                        (const uint2 *)(base + o_iC),
+                        (const uint2 *)(base + o_iCR)};
     e = (cudaError_t)launch_phases(a, lp, stream, nullptr);
     if (e != cudaSuccess) return SKEW_ECUDA;
     return SKEW_OK;

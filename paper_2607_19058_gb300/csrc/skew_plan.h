@@ -142,18 +142,19 @@ struct StepArgs {
 //   F  finalize items (rows and columns; columns only on the row path)
 //   B  update-RMS tiles (strip-path factored and full tensors)
 //   FB phase B of the row-path tensors whose finalize asked for it (nFB CTAs)
-//   C  apply tiles (every tensor)
+//   C  apply strip tiles (tensors not on the row path)
+//   CR apply row tiles (row-path tensors)
 struct LaunchPlan {
-    uint32_t nA, nR, nF, nB, nFB, nC;
-    const uint2 *itemsA, *itemsR, *itemsF, *itemsB, *itemsC;
+    uint32_t nA, nR, nF, nB, nFB, nC, nCR;
+    const uint2 *itemsA, *itemsR, *itemsF, *itemsB, *itemsC, *itemsCR;
 };
 
-constexpr int kLaunches = 6;
+constexpr int kLaunches = 7;
 
-// Enqueues the phases of `L` as grouped launches (A, R, F, B, FB, C; empty ones
-// skipped) on `stream`, each given the step parameters by value. If `ev` is not
-// null it holds kLaunches + 1 cudaEvent_t, recorded before the first launch and
-// after each of the six. Returns a cudaError_t value.
+// Enqueues the phases of `L` as grouped launches (A, R, F, B, FB, C, CR; empty
+// ones skipped) on `stream`, each given the step parameters by value. If `ev` is
+// not null it holds kLaunches + 1 cudaEvent_t, recorded before the first launch
+// and after each of the seven. Returns a cudaError_t value.
 int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *const *ev);
 
 }  // namespace skew
