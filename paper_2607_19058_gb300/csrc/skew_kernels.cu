@@ -496,21 +496,25 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(b)), "r"(bytes) : "memory");
 }
 
+// One poll; the thread may be suspended for up to about kMbarSuspendNs while the
+// phase is incomplete (a hint to the hardware).
+constexpr uint32_t kMbarSuspendNs = 2000;
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *b, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(smem_u32(b)), "r"(parity)
+        : "r"(smem_u32(b)), "r"(parity), "n"(kMbarSuspendNs)
         : "memory");
     return ok != 0;
 }
 
-// Polls of one mbarrier wait before it gives up (each poll may suspend the
-// thread for a short hardware-defined time): a copy that never lands ends the
-// tile with a status word instead of hanging the GPU.
+// Polls of one mbarrier wait before it gives up (about two seconds at the
+// suspend hint): a copy that never lands ends the tile with a status word
+// instead of hanging the GPU.
 constexpr uint32_t kMbarPolls = 1u << 20;
 
 __device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
@@ -761,6 +765,23 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
     }
 }
 
+// sum_{r < cnt} p[r * stride] (values an earlier launch wrote), added in order
+// r = 0, 1, ...; the loads are issued eight at a time ahead of the adds.
+template <typename V>
+__device__ __forceinline__ V strided_sum(const V *p, int64_t stride, uint32_t cnt) {
+    V s = V(0);
+    uint32_t r = 0;
+    for (; r + 8 <= cnt; r += 8) {
+        V v[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) v[q] = __ldcg(p + int64_t(r + q) * stride);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) s += v[q];
+    }
+    for (; r < cnt; ++r) s += __ldcg(p + int64_t(r) * stride);
+    return s;
+}
+
 // mean(R) and its [1, 2) mantissa / exponent split (used by the row scales).
 __device__ void set_rbar(TensorScal &S, double rbar) {
     S.rbar = rbar;
@@ -801,12 +822,8 @@ __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem 
     double contrib = 0.0;
     float cmin = inf;
     if (threadIdx.x < kFinChunk && j < T.m) {
-        float cs = 0.f;
-        double P = 0.0;
-        for (uint32_t r = 0; r < T.rtiles; ++r) {
-            cs += __ldcg(T.colp + int64_t(r) * T.m + j);
-            P += __ldcg(T.pp + int64_t(r) * T.m + j);
-        }
+        const float cs = strided_sum(T.colp + j, T.m, T.rtiles);
+        const double P = strided_sum(T.pp + j, T.m, T.rtiles);
         const float mean = __fdiv_rn(cs, (float)T.n);
         const float Cn = fmaf(A.b2, T.C[j], A.c2 * mean);
         T.C[j] = Cn;
@@ -874,8 +891,7 @@ __device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm)
         const int64_t i = int64_t(local) * kFinChunk + threadIdx.x;
         double rd = 0.0;
         if (threadIdx.x < kFinChunk && i < T.n) {
-            float rs = 0.f;
-            for (uint32_t s = 0; s < T.strips; ++s) rs += __ldcg(T.rowp + int64_t(s) * T.n + i);
+            const float rs = strided_sum(T.rowp + i, T.n, T.strips);
             const float mean = __fdiv_rn(rs, (float)T.m);
             const float Rn = fmaf(A.b2, T.R[i], A.c2 * mean);
             T.R[i] = Rn;
@@ -886,8 +902,7 @@ __device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm)
     } else {
         const int64_t j = int64_t(local - T.nfr) * kFinChunk + threadIdx.x;
         if (threadIdx.x < kFinChunk && j < T.m) {
-            float cs = 0.f;
-            for (uint32_t r = 0; r < T.rowtiles; ++r) cs += __ldcg(T.colp + int64_t(r) * T.m + j);
+            const float cs = strided_sum(T.colp + j, T.m, T.rowtiles);
             const float mean = __fdiv_rn(cs, (float)T.n);
             const float Cn = fmaf(A.b2, T.C[j], A.c2 * mean);
             T.C[j] = Cn;
