@@ -276,6 +276,25 @@ METRIC = "SkewAdam optimizer step over the 6.78B-parameter MoE shape set: params
 
 
 # ---------------------------------------------------------------------------
+# Across ranks (one process per GPU; every rank steps its own full parameter set)
+# ---------------------------------------------------------------------------
+def max_over_ranks(x, world, device):
+    """The largest `x` over the ranks (the job's time is its slowest rank's); `x` on one rank."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, params_per_rank, ms):
+    """Whole-job parameters per second: every rank's parameters over the job's step time."""
+    return world * params_per_rank / (ms * 1e-3)
+
+
+# ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
 def run_ours(args):
@@ -325,11 +344,8 @@ def run_ours(args):
     clocks = clocks_stop(clk)
     opt.sync_status()
     names, rows = S.skew_profile_end(opt.h)
-    ms = e0.elapsed_time(e1) / args.steps
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world, dev)
     if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
         dist.barrier()
 
     # per-kernel live durations
@@ -367,12 +383,8 @@ def run_ours(args):
                 views[k][1].copy_(W[k], non_blocking=True)
         b.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = a.elapsed_time(b) / args.e2e_steps
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
-        e2e = {"value": world * bm["N"] / (e2e_ms * 1e-3), "unit": "params/s", "ms_per_step": e2e_ms,
+        e2e_ms = max_over_ranks(a.elapsed_time(b) / args.e2e_steps, world, dev)
+        e2e = {"value": job_rate(world, bm["N"], e2e_ms), "unit": "params/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": 2 * bm["N"], "d2h_bytes_per_step": 2 * bm["N"],
                "path": "skew_step via ctypes; gradients copied in from pinned host memory and weights read back "
                        "to pinned host memory every step"}
@@ -392,7 +404,7 @@ def run_ours(args):
     if rank == 0:
         out = {
             "metric": METRIC,
-            "value": world * bm["N"] / (ms * 1e-3), "unit": "params/s", "n_gpus": world, "steps": args.steps,
+            "value": job_rate(world, bm["N"], ms), "unit": "params/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {"workload": wl.name, "params": bm["N"], "tensors": len(wl.specs), "policy": "tiered",
