@@ -213,6 +213,13 @@ __device__ __forceinline__ void two_sum2(float2 a, float2 b, float2 &s, float2 &
     e = __fadd2_rn(__fadd2_rn(a, neg2(__fadd2_rn(s, neg2(bp)))), __fadd2_rn(b, neg2(bp)));
 }
 
+// The value of a compensated (hi, lo) pair in fp64. Once an infinite term has
+// entered, TwoSum's error term is NaN (inf - inf) while hi carries the sum
+// (+-inf, or NaN for inf - inf), so a non-finite hi is the value on its own.
+__device__ __forceinline__ double pair_value(float hi, float lo) {
+    return isfinite(hi) ? (double)hi + (double)lo : (double)hi;
+}
+
 // Compensated accumulator: the running sum is hi + lo.
 struct Acc2 {
     float hi = 0.f, lo = 0.f;
@@ -749,7 +756,7 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         double2 *pp2 = reinterpret_cast<double2 *>(T.pp + base + col);
 #pragma unroll
         for (int q = 0; q < 4; ++q)
-            pp2[q] = make_double2((double)ph[v][q].x + (double)pl[v][q].x, (double)ph[v][q].y + (double)pl[v][q].y);
+            pp2[q] = make_double2(pair_value(ph[v][q].x, pl[v][q].x), pair_value(ph[v][q].y, pl[v][q].y));
     }
     if (zero_row) atomicOr(&S.zflag, 1u);
     if (warp == 0) {
@@ -1059,7 +1066,7 @@ __device__ void phase_B(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm,
     double s = 0.0;
     for (uint32_t k = threadIdx.x; k < T.ntiles; k += kThreads) {
         const float2 p = __ldcg(T.u2 + k);
-        s += (double)p.x + (double)p.y;
+        s += pair_value(p.x, p.y);
     }
     s = block_sum_d(s, sm.redd);
     if (threadIdx.x == 0) set_clip(A, T, S, s);
