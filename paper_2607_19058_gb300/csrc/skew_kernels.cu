@@ -548,11 +548,17 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 
 __device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
 
+// Threads of the row-path kernels (256 or 512).
+#ifndef SKEW_ROW_THREADS
+#define SKEW_ROW_THREADS 256
+#endif
+constexpr int kRowThreads = SKEW_ROW_THREADS;
+
 struct RowSmem {
     uint4 buf[kRowStages][kRowChunkBytes / 16];  // the chunk ring (first member: 16-byte aligned)
     uint64_t full[kRowStages];                   // one mbarrier per ring slot
-    float part[kThreads / 32][8];                // per-warp row partial sums of the chunk
-    float inv[8];                                // 1 / R_i of the chunk's rows (0: no contribution)
+    float part[kRowThreads / 32][8];             // per-warp row partial sums of the chunk
+    float inv[32];                               // 1 / R_i of the chunk's rows (0: no contribution)
     int fail;
 };
 
@@ -617,11 +623,29 @@ __device__ __forceinline__ void row_issue(const TensorDev &T, uint32_t tile, uin
     bulk_g2s(sm.buf[st], T.g + ch.i0 * T.m, bytes, &sm.full[st], pol);
 }
 
-// NV 16-byte vectors per thread per row (m = 2048 * NV), CR = 8 / NV rows per chunk.
-template <int NV>
+// Thread layout of a row-path kernel with TPB threads on rows of V = m / 8
+// 16-byte vectors: NV vectors per thread per row (V > TPB), or RPP rows side by side
+// (V < TPB); a thread owns vectors vi, vi + TPB, ... of row-in-pass rp.
+template <int TPB, int V>
+struct RowLayout {
+    static constexpr int NV = V > TPB ? V / TPB : 1;
+    static constexpr int RPP = V < TPB ? TPB / V : 1;
+    static constexpr int WPR = (V < TPB ? V : TPB) / 32;  // warps per row-in-pass
+    int rp, vi;
+    __device__ RowLayout() : rp(threadIdx.x / (V < TPB ? V : TPB)), vi(threadIdx.x % (V < TPB ? V : TPB)) {}
+};
+
+// k_rowsq on TPB threads, rows of m = 8 V: chunks of CS = 2048 / V rows (32 KB),
+// K = CS / RPP rows per thread per chunk.
+template <int TPB, int V>
 __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S, uint32_t tile, RowSmem &sm) {
-    constexpr int CR = 8 / NV;
-    constexpr int V = kThreads * NV;  // vectors per row
+    using L = RowLayout<TPB, V>;
+    constexpr int NV = L::NV, RPP = L::RPP, WPR = L::WPR;
+    constexpr int CS = 2048 / V;
+    constexpr int K = CS / RPP;
+    static_assert(K == 4 || K == 8, "rows per thread per chunk");
+    static_assert(CS <= 32, "chunk rows");
+    const L lay;
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
     const uint32_t nch = (uint32_t)min((int64_t)kRowChunks, (T.n - int64_t(tile) * T.rt_rows + T.cr - 1) / T.cr);
@@ -635,15 +659,15 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         for (uint32_t c = 0; c < nch && c < (uint32_t)kRowStages; ++c) row_issue(T, tile, c, sm, pol);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const float b2 = A.b2, c2 = A.c2, fm = (float)T.m;
+    const float b2 = A.b2, c2 = A.c2, inv_m = 1.0f / (float)(8 * V);  // m is a power of two: exact
     // per column pair: sums of g^2 and the compensated (hi, lo) sum of g^2 / R_i
     float2 cs[NV][4], ph[NV][4], pl[NV][4];
 #pragma unroll
     for (int v = 0; v < NV; ++v)
 #pragma unroll
         for (int q = 0; q < 4; ++q) cs[v][q] = ph[v][q] = pl[v][q] = make_float2(0.f, 0.f);
-    double rsum = 0.0;                       // threads < CR: sum of this lane's rows' R
-    float rmin = __int_as_float(0x7F800000);  // threads < CR: smallest positive R of this lane's rows
+    double rsum = 0.0;                       // threads < CS: sum of the R of this chunk-row position
+    float rmin = __int_as_float(0x7F800000);  // threads < CS: smallest positive R of it
     bool zero_row = false;
 
     uint32_t c = 0;
@@ -655,16 +679,17 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         if (tid < (int)ch.rows) rp = __ldcg(T.R + ch.i0 + tid);
         const bool ok = mbar_wait(&sm.full[st], par);
         const uint4 *buf = sm.buf[st];
-        // pass 1: row sums and column sums of g^2
-        float rs[CR];
+        // pass 1: row sums and column sums of g^2 (rows lay.rp + RPP k of the chunk)
+        float rs[K];
 #pragma unroll
-        for (int r = 0; r < CR; ++r) {
+        for (int k = 0; k < K; ++k) {
+            const int r = lay.rp + RPP * k;
             float2 r2 = make_float2(0.f, 0.f);
             if (r < (int)ch.rows) {
 #pragma unroll
                 for (int v = 0; v < NV; ++v) {
                     float2 g[4];
-                    unpack_bf8x2(buf[r * V + v * kThreads + tid], g);
+                    unpack_bf8x2(buf[r * V + v * TPB + lay.vi], g);
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
                         const float2 sq = __fmul2_rn(g[q], g[q]);
@@ -673,22 +698,23 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
                     }
                 }
             }
-            rs[r] = r2.x + r2.y;
+            rs[k] = r2.x + r2.y;
         }
         int j;
-        const float tot = warp_sum_transposed<CR>(rs, j);
-        if ((lane & (CR == 8 ? 3 : 7)) == 0) sm.part[warp][j] = tot;
+        const float tot = warp_sum_transposed<K>(rs, j);
+        if ((lane & (K == 8 ? 3 : 7)) == 0) sm.part[warp][j] = tot;
         if (__syncthreads_or(!ok)) break;  // every slot before this one has landed
         // slot of chunk c - 1 is free (its pass 2 preceded this barrier): refill it
         if (tid == 0 && c >= 1 && c - 1 + kRowStages < nch) {
             fence_proxy_async_smem();
             row_issue(T, tile, c - 1 + kRowStages, sm, pol);
         }
-        if (tid < (int)ch.rows) {
+        if (tid < (int)ch.rows) {  // chunk row r = tid: row-in-pass r % RPP, its k = r / RPP
+            const int w0 = (tid % RPP) * WPR, kr = tid / RPP;
             float sum = 0.f;
 #pragma unroll
-            for (int w = 0; w < kThreads / 32; ++w) sum += sm.part[w][tid];
-            const float mean = __fdiv_rn(sum, fm);
+            for (int w = 0; w < WPR; ++w) sum += sm.part[w0 + w][kr];
+            const float mean = sum * inv_m;
             const float Rn = fmaf(b2, rp, c2 * mean);
             T.R[ch.i0 + tid] = Rn;
             rsum += (double)Rn;
@@ -709,14 +735,15 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
 #pragma unroll
             for (int q = 0; q < 4; ++q) t[v][q] = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int r = 0; r < CR; ++r) {
+        for (int k = 0; k < K; ++k) {
+            const int r = lay.rp + RPP * k;
             if (r < (int)ch.rows) {
                 const float iv = sm.inv[r];
                 const float2 iv2 = make_float2(iv, iv);
 #pragma unroll
                 for (int v = 0; v < NV; ++v) {
                     float2 g[4];
-                    unpack_bf8x2(buf[r * V + v * kThreads + tid], g);
+                    unpack_bf8x2(buf[r * V + v * TPB + lay.vi], g);
 #pragma unroll
                     for (int q = 0; q < 4; ++q) t[v][q] = __ffma2_rn(__fmul2_rn(g[q], g[q]), iv2, t[v][q]);
                 }
@@ -744,22 +771,49 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         }
         return;
     }
-    // per-tile partials: column sums of g^2 and of g^2 / R_i, the tile's sum and
-    // smallest positive R
-    const int64_t base = int64_t(tile) * T.m;
+    // per-tile partials: column sums of g^2 and of g^2 / R_i (the RPP threads that share
+    // a column vector are added in row-in-pass order), the tile's sum and smallest positive R
+    const int64_t base = int64_t(tile) * 8 * V;
+    if constexpr (RPP == 1) {
 #pragma unroll
-    for (int v = 0; v < NV; ++v) {
-        const int64_t col = 8 * int64_t(v * kThreads + tid);
-        float4 *cp4 = reinterpret_cast<float4 *>(T.colp + base + col);
-        cp4[0] = make_float4(cs[v][0].x, cs[v][0].y, cs[v][1].x, cs[v][1].y);
-        cp4[1] = make_float4(cs[v][2].x, cs[v][2].y, cs[v][3].x, cs[v][3].y);
-        double2 *pp2 = reinterpret_cast<double2 *>(T.pp + base + col);
+        for (int v = 0; v < NV; ++v) {
+            const int64_t col = 8 * int64_t(v * TPB + lay.vi);
+            float4 *cp4 = reinterpret_cast<float4 *>(T.colp + base + col);
+            cp4[0] = make_float4(cs[v][0].x, cs[v][0].y, cs[v][1].x, cs[v][1].y);
+            cp4[1] = make_float4(cs[v][2].x, cs[v][2].y, cs[v][3].x, cs[v][3].y);
+            double2 *pp2 = reinterpret_cast<double2 *>(T.pp + base + col);
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-            pp2[q] = make_double2(pair_value(ph[v][q].x, pl[v][q].x), pair_value(ph[v][q].y, pl[v][q].y));
+            for (int q = 0; q < 4; ++q)
+                pp2[q] = make_double2(pair_value(ph[v][q].x, pl[v][q].x), pair_value(ph[v][q].y, pl[v][q].y));
+        }
+    } else {
+        // the ring is free (every chunk consumed before the last barrier): stage there
+        float *mcs = reinterpret_cast<float *>(sm.buf[0]);        // [TPB][8]
+        double *mpp = reinterpret_cast<double *>(sm.buf[1]);      // [TPB][8]
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            mcs[tid * 8 + 2 * q] = cs[0][q].x;
+            mcs[tid * 8 + 2 * q + 1] = cs[0][q].y;
+            mpp[tid * 8 + 2 * q] = pair_value(ph[0][q].x, pl[0][q].x);
+            mpp[tid * 8 + 2 * q + 1] = pair_value(ph[0][q].y, pl[0][q].y);
+        }
+        __syncthreads();
+        for (int e = tid; e < 8 * V; e += TPB) {  // column e = 8 vi + q
+            const int vi = e >> 3, q = e & 7;
+            float cc = 0.f;
+            double pq = 0.0;
+#pragma unroll
+            for (int r = 0; r < RPP; ++r) {
+                cc += mcs[(r * V + vi) * 8 + q];
+                pq += mpp[(r * V + vi) * 8 + q];
+            }
+            T.colp[base + e] = cc;
+            T.pp[base + e] = pq;
+        }
     }
     if (zero_row) atomicOr(&S.zflag, 1u);
-    if (warp == 0) {
+    if (warp == 0) {  // CS <= 32: the chunk-row positions are lanes of warp 0
 #pragma unroll
         for (int o = 16; o; o >>= 1) {
             rsum += __shfl_xor_sync(kAll, rsum, o);
@@ -1238,8 +1292,8 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
 struct ApplyRowSmem {
     uint4 buf[kRowStages][kRowChunkBytes / 16];  // [W rows | G rows] per slot
     uint64_t full[kRowStages];
-    float a[kRowChunks * 8];                     // row scales a_i of the tile (rt_rows <= 256)
-    float red[2 * kThreads / 32];
+    float a[kRowChunks * 32];                    // row scales a_i of the tile (rt_rows <= 1024)
+    float red[2 * kRowThreads / 32];
 };
 
 __device__ __forceinline__ void apply_row_issue(const TensorDev &T, uint32_t tile, uint32_t c, uint32_t ca,
@@ -1253,13 +1307,17 @@ __device__ __forceinline__ void apply_row_issue(const TensorDev &T, uint32_t til
     bulk_g2s(sm.buf[st] + kRowChunkBytes / 32, T.g + i0 * T.m, bytes, &sm.full[st], pol);
 }
 
-template <int NV, bool FAST>
-__device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t tile, const float (&b)[NV][8],
-                                float coefC, ApplyRowSmem &sm, uint32_t nch, uint32_t ca, uint64_t pol) {
-    constexpr int V = kThreads * NV;       // vectors per row
-    constexpr int CA = 4 / NV;             // rows per chunk (16 KB of W, 16 KB of G)
+// CA = 1024 / V rows per chunk (16 KB of W, 16 KB of G), KA = CA / RPP rows per thread.
+template <int TPB, int V, bool FAST>
+__device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t tile,
+                                const float (&b)[RowLayout<TPB, V>::NV][8], float coefC, ApplyRowSmem &sm,
+                                uint32_t nch, uint64_t pol) {
+    using L = RowLayout<TPB, V>;
+    constexpr int NV = L::NV, RPP = L::RPP;
+    constexpr int CA = 1024 / V, KA = CA / RPP;
+    const L lay;
     const int tid = threadIdx.x;
-    const int64_t m = T.m;
+    const int64_t m = 8 * V;
     uint16_t *__restrict__ w_ = T.w;
     const Dith d = dith_of(A, T.tid);
     const float wdf = T.decay ? A.wdf : 1.0f;
@@ -1268,13 +1326,14 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
     const Pol sp;
     for (uint32_t c = 0; c < nch; ++c) {
         const int st = c % kRowStages;
-        const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * ca;
+        const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * CA;
         const int rows = (int)min((int64_t)CA, T.n - i0);
         const bool ok = mbar_wait(&sm.full[st], (c / kRowStages) & 1u);
         const uint4 *bw = sm.buf[st];
         const uint4 *bg = sm.buf[st] + kRowChunkBytes / 32;
 #pragma unroll
-        for (int r = 0; r < CA; ++r) {
+        for (int k = 0; k < KA; ++k) {
+            const int r = lay.rp + RPP * k;
             if (r < rows) {
                 const float a = sm.a[c * CA + r];
                 const float cr = -coefC * a;
@@ -1282,8 +1341,8 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
 #pragma unroll
                 for (int v = 0; v < NV; ++v) {
                     float y[8], w[8], x[8];
-                    unpack_bf8(bg[r * V + v * kThreads + tid], y);
-                    unpack_bf8(bw[r * V + v * kThreads + tid], w);
+                    unpack_bf8(bg[r * V + v * TPB + lay.vi], y);
+                    unpack_bf8(bw[r * V + v * TPB + lay.vi], w);
                     if constexpr (FAST) {
 #pragma unroll
                         for (int q = 0; q < 4; ++q) {
@@ -1296,9 +1355,9 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
                         }
                     } else {
 #pragma unroll
-                        for (int k = 0; k < 8; ++k) x[k] = fmaf(-coefC, y[k] * fminf(a * b[v][k], ce), w[k] * wdf);
+                        for (int q = 0; q < 8; ++q) x[q] = fmaf(-coefC, y[q] * fminf(a * b[v][q], ce), w[q] * wdf);
                     }
-                    write8<true>(w_, d, (i0 + r) * m + 8 * (v * kThreads + tid), 8, true, x, sp);
+                    write8<true>(w_, d, (i0 + r) * m + 8 * (v * TPB + lay.vi), 8, true, x, sp);
                 }
             }
         }
@@ -1314,15 +1373,18 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
         }
         if (tid == 0 && c + kRowStages < nch) {
             fence_proxy_async_smem();
-            apply_row_issue(T, tile, c + kRowStages, ca, sm, pol);
+            apply_row_issue(T, tile, c + kRowStages, CA, sm, pol);
         }
     }
 }
 
-template <int NV>
+template <int TPB, int V>
 __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile,
                                 ApplyRowSmem &sm) {
-    constexpr int CA = 4 / NV;
+    using L = RowLayout<TPB, V>;
+    constexpr int NV = L::NV;
+    constexpr int CA = 1024 / V;
+    const L lay;
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
     const int64_t r0 = int64_t(tile) * T.rt_rows;
@@ -1339,7 +1401,7 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
     const float rbar_s = __ldcg(&S.rbar_s);
     const int rbar_e = __ldcg(&S.rbar_e);
     float ma = 0.f, mb = 0.f;
-    for (uint32_t r = threadIdx.x; r < rows_t; r += kThreads) {
+    for (uint32_t r = threadIdx.x; r < rows_t; r += TPB) {
         const float a = row_scale(__ldcg(T.R + r0 + r), rbar_s, rbar_e);
         sm.a[r] = a;
         ma = fmaxf(ma, nan_to_inf(a));
@@ -1347,7 +1409,7 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
     float b[NV][8];
 #pragma unroll
     for (int v = 0; v < NV; ++v) {
-        const float *p = T.bsc + 8 * (v * kThreads + threadIdx.x);
+        const float *p = T.bsc + 8 * (v * TPB + lay.vi);
         const float4 b0 = __ldcg(reinterpret_cast<const float4 *>(p));
         const float4 b1 = __ldcg(reinterpret_cast<const float4 *>(p + 4));
         b[v][0] = b0.x; b[v][1] = b0.y; b[v][2] = b0.z; b[v][3] = b0.w;
@@ -1362,20 +1424,20 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
     }
     if ((threadIdx.x & 31) == 0) {
         sm.red[threadIdx.x >> 5] = ma;
-        sm.red[kThreads / 32 + (threadIdx.x >> 5)] = mb;
+        sm.red[TPB / 32 + (threadIdx.x >> 5)] = mb;
     }
     __syncthreads();
     ma = mb = 0.f;
 #pragma unroll
-    for (int w = 0; w < kThreads / 32; ++w) {
+    for (int w = 0; w < TPB / 32; ++w) {
         ma = fmaxf(ma, sm.red[w]);
-        mb = fmaxf(mb, sm.red[kThreads / 32 + w]);
+        mb = fmaxf(mb, sm.red[TPB / 32 + w]);
     }
     const float coefC = __ldcg(&S.coefC);
     if (ma * mb <= A.ce)
-        apply_rows_body<NV, true>(A, T, tile, b, coefC, sm, nch, CA, pol);
+        apply_rows_body<TPB, V, true>(A, T, tile, b, coefC, sm, nch, pol);
     else
-        apply_rows_body<NV, false>(A, T, tile, b, coefC, sm, nch, CA, pol);
+        apply_rows_body<TPB, V, false>(A, T, tile, b, coefC, sm, nch, pol);
 }
 
 // ---------------------------------------------------------------------------
@@ -1396,28 +1458,35 @@ __global__ void __launch_bounds__(kThreads, SKEW_MINB_SUMSQ)
 }
 
 // Row path, phase A: one row tile per CTA (dynamic shared memory: RowSmem).
-__global__ void __launch_bounds__(kThreads, 2) k_rowsq(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
+__global__ void __launch_bounds__(kRowThreads, 512 / kRowThreads)
+    k_rowsq(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
     extern __shared__ uint4 dyn_smem[];
     RowSmem &sm = *reinterpret_cast<RowSmem *>(dyn_smem);
     const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
-    if (T.m == 4096)
-        rowsq_tile<2>(A, T, A.scal[it.x], it.y, sm);
-    else
-        rowsq_tile<1>(A, T, A.scal[it.x], it.y, sm);
+    TensorScal &S = A.scal[it.x];
+    switch (T.m) {
+        case 4096: rowsq_tile<kRowThreads, 512>(A, T, S, it.y, sm); break;
+        case 2048: rowsq_tile<kRowThreads, 256>(A, T, S, it.y, sm); break;
+        case 1024: rowsq_tile<kRowThreads, 128>(A, T, S, it.y, sm); break;
+        default: rowsq_tile<kRowThreads, 64>(A, T, S, it.y, sm); break;  // 512
+    }
 }
 
 // Row path, phase C: one row tile per CTA (dynamic shared memory: ApplyRowSmem).
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kRowThreads, 512 / kRowThreads)
     k_apply_rows(const __grid_constant__ StepArgs A, const uint2 *__restrict__ items) {
     extern __shared__ uint4 dyn_smem[];
     ApplyRowSmem &sm = *reinterpret_cast<ApplyRowSmem *>(dyn_smem);
     const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
-    if (T.m == 4096)
-        apply_rows_tile<2>(A, T, A.scal[it.x], it.y, sm);
-    else
-        apply_rows_tile<1>(A, T, A.scal[it.x], it.y, sm);
+    const TensorScal &S = A.scal[it.x];
+    switch (T.m) {
+        case 4096: apply_rows_tile<kRowThreads, 512>(A, T, S, it.y, sm); break;
+        case 2048: apply_rows_tile<kRowThreads, 256>(A, T, S, it.y, sm); break;
+        case 1024: apply_rows_tile<kRowThreads, 128>(A, T, S, it.y, sm); break;
+        default: apply_rows_tile<kRowThreads, 64>(A, T, S, it.y, sm); break;  // 512
+    }
 }
 
 // Phase B of the row-path tensors whose finalize found that a clamp may bind
@@ -1503,7 +1572,7 @@ int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *co
     if (L.nR) {
         const cudaError_t e = cudaFuncSetAttribute(k_rowsq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RowSmem));
         if (e != cudaSuccess) return (int)e;
-        k_rowsq<<<L.nR, kThreads, sizeof(RowSmem), s>>>(A, L.itemsR);
+        k_rowsq<<<L.nR, kRowThreads, sizeof(RowSmem), s>>>(A, L.itemsR);
     }
     mark(2);
     if (L.nF) k_finalize<<<L.nF, kThreads, 0, s>>>(A, L.itemsF);
@@ -1518,7 +1587,7 @@ int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *co
         const cudaError_t e =
             cudaFuncSetAttribute(k_apply_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(ApplyRowSmem));
         if (e != cudaSuccess) return (int)e;
-        k_apply_rows<<<L.nCR, kThreads, sizeof(ApplyRowSmem), s>>>(A, L.itemsCR);
+        k_apply_rows<<<L.nCR, kRowThreads, sizeof(ApplyRowSmem), s>>>(A, L.itemsCR);
     }
     mark(7);
     return (int)cudaGetLastError();

@@ -50,9 +50,9 @@ inline TileGeom plan_geometry(uint32_t kind, uint32_t momentum, bool wg_aligned,
         g.rowtiles = (uint32_t)((n + g.tile_rows - 1) / g.tile_rows);
         g.ntiles = g.strips * g.rowtiles;
         g.nfc = (uint32_t)((m + kFinChunk - 1) / kFinChunk);
-        // Whole-row phase A: momentum-free factored matrices of width 2048 or
-        // 4096 (one or two 16-byte vectors per thread per row).
-        g.rowpath = (!momentum && wg_aligned && (m == 2048 || m == 4096)) ? 1u : 0u;
+        // Whole-row phases A and C: momentum-free factored matrices of width
+        // 512, 1024, 2048 or 4096 (64 to 512 16-byte vectors per row).
+        g.rowpath = (!momentum && wg_aligned && (m == 512 || m == 1024 || m == 2048 || m == 4096)) ? 1u : 0u;
         if (g.rowpath) {
             g.cr = (uint32_t)(kRowChunkBytes / (2 * m));
             g.rt_rows = g.cr * kRowChunks;

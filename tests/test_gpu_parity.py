@@ -198,11 +198,13 @@ def test_ablation_awkward_full_size_subset():
 
 
 def _row_path_workload():
-    """Momentum-free matrices of width 4096 / 2048 (the whole-row phase A): ragged
-    row tiles and chunks, and expert 5 with zero gradients on odd steps."""
+    """Momentum-free matrices of width 4096 / 2048 / 1024 / 512 (the whole-row
+    phases A and C): ragged row tiles and chunks, and expert 5 with zero gradients on
+    odd steps."""
     E = WL.TIER_EXPERT
     specs = [WL.Spec("e512x4096", (512, 4096), E, expert=0), WL.Spec("e301x4096", (301, 4096), E, expert=1),
              WL.Spec("e1000x2048", (1000, 2048), E, expert=2), WL.Spec("e77x2048", (77, 2048), E, expert=3),
+             WL.Spec("e1333x1024", (1333, 1024), E, expert=4), WL.Spec("e2101x512", (2101, 512), E, expert=6),
              WL.Spec("zero_odd", (256, 4096), E, expert=5)]
     return WL.Workload("rowpath", specs, WL.HP(), "toy", steps=4)
 
