@@ -87,11 +87,18 @@ typedef struct skew_handle skew_handle_t; /* opaque */
  *   grad   : device pointer to the bf16 gradient, same shape and layout; read
  *            only. Borrowed like `weight`.
  *   shape  : shape[0] = rows n (>= 1); shape[1] = columns m (>= 1) when
- *            ndim == 2, ignored when ndim == 1.
- *   ndim   : 1 (vector) or 2 (matrix).
+ *            ndim >= 2, ignored when ndim == 1.
+ *   ndim   : 1 (vector), 2 (matrix) or 3 (a stack of `stack` matrices of
+ *            n x m, contiguous: matrix e starts at element e*n*m).
  *   tier   : SKEW_TIER_*.
  *   flags  : SKEW_F_* bits.
- *   reserved: must be 0.
+ *   stack  : the number of matrices when ndim == 3 (>= 1); 0 otherwise.
+ *
+ * A stacked tensor (experts kept as one (E, n, m) array) is stepped as E
+ * matrices, each with its own second-moment factors, RMS and clip factor
+ * (Algorithm 1 is stated per matrix; the paper counts 128 x 3 expert
+ * matrices); its dither uses the descriptor's index as tensor id and the flat
+ * index e*n*m + i*m + j over the whole stack.
  */
 typedef struct {
     void *weight;
@@ -100,7 +107,7 @@ typedef struct {
     int32_t ndim;
     int32_t tier;
     uint32_t flags;
-    uint32_t reserved;
+    uint32_t stack;
 } skew_param_desc_t;
 
 /*
@@ -134,7 +141,9 @@ typedef struct {
     int64_t m_offset, v_offset, r_offset, c_offset;
     int32_t rowpath;    /* 1 if phase A runs on whole rows and sum(U^2) needs no  */
                         /* second pass over G unless a clamp may bind (bilinear) */
-    int32_t reserved;   /* 0                                                   */
+    int32_t stack;      /* matrices of a stacked tensor (ndim 3), else 0; then   */
+                        /* rows / cols are one matrix's, numel the whole stack's, */
+                        /* and each state array holds the E matrices' in order   */
 } skew_tensor_info_t;
 
 /*
@@ -206,6 +215,10 @@ int skew_sync_status(skew_handle_t *h, void *stream);
  * `stream`. Errors: SKEW_EINVAL (tid), SKEW_ESTATE, SKEW_ECUDA.
  */
 int skew_tensor_scalars(skew_handle_t *h, int32_t tid, double out[4], void *stream);
+
+/* As skew_tensor_scalars, for matrix `e` of stacked tensor `tid` (e = 0 for any
+ * other tensor). Errors: SKEW_EINVAL (tid, e), SKEW_ESTATE, SKEW_ECUDA. */
+int skew_matrix_scalars(skew_handle_t *h, int32_t tid, int32_t e, double out[4], void *stream);
 
 /* Resolved policy and state offsets of tensor `tid`. Errors: SKEW_EINVAL. */
 int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *out);

@@ -46,6 +46,7 @@ class _Tensor(C.Structure):
         ("w", C.c_void_p), ("g", C.c_void_p), ("M", C.c_void_p), ("v", C.c_void_p),
         ("R", C.c_void_p), ("C", C.c_void_p), ("n", C.c_int64), ("m", C.c_int64),
         ("kind", C.c_int32), ("momentum", C.c_int32), ("decay", C.c_int32), ("tid", C.c_uint32),
+        ("idx0", C.c_uint64),
     ]
 
 
@@ -156,7 +157,7 @@ def hparams(beta1, beta2, eps, clip_d, weight_decay):
 
 
 def tensor_step(w_bits: np.ndarray, g_bits: np.ndarray, st: TensorState, tid: int, hp, step: int,
-                lr: float, seed: int, want_x: bool = False):
+                lr: float, seed: int, want_x: bool = False, idx0: int = 0):
     """One oracle step of one tensor; `w_bits` (uint16) and the state update in place.
 
     Returns a dict with Rbar, sum of U^2, RMS and kappa, plus the fp32 pre-rounding
@@ -167,7 +168,7 @@ def tensor_step(w_bits: np.ndarray, g_bits: np.ndarray, st: TensorState, tid: in
     numel = st.n * st.m
     assert w_bits.size == numel and g_bits.size == numel
     T = _Tensor(_ptr(w_bits), _ptr(g_bits), _ptr(st.M), _ptr(st.v), _ptr(st.R), _ptr(st.C),
-                st.n, st.m, st.kind, st.momentum, st.decay, tid)
+                st.n, st.m, st.kind, st.momentum, st.decay, tid, idx0)
     x = np.empty(numel, np.float32) if want_x else None
     r = np.empty(numel, np.uint16) if want_x else None
     stats = np.zeros(4, np.float64)

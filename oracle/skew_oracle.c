@@ -225,6 +225,8 @@ typedef struct {
     int32_t momentum;   /* 1: keeps fp32 momentum                                */
     int32_t decay;      /* 1: weight decay applies                               */
     uint32_t tid;       /* tensor id fed to the dither                           */
+    uint64_t idx0;      /* dither index of element 0: 0, or for matrix e of a    */
+                        /* stacked (E, n, m) tensor e*n*m (its flat offset)      */
 } so_tensor_t;
 
 typedef struct {
@@ -308,7 +310,7 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
     for (int64_t e = 0; e < numel; ++e) {
         double w = so_bf16_to_double(T->w[e]);
         float x = (float)(w * (1.0 - lr * lam) - lr * kappa * U[e]);
-        uint16_t r = so_dither16(seed, t, T->tid, (uint64_t)e);
+        uint16_t r = so_dither16(seed, t, T->tid, T->idx0 + (uint64_t)e);
         T->w[e] = so_sr_bf16(x, r);
         if (x_out) x_out[e] = x;
         if (r_out) r_out[e] = r;

@@ -24,7 +24,12 @@ using namespace skew;
 
 namespace {
 
+// One matrix or vector stepped on its own (a stacked descriptor gives several).
 struct TPlan {
+    void *w = nullptr;        // its bf16 weights and gradient
+    const void *g = nullptr;
+    uint32_t tid = 0;         // the descriptor's index: the dither's tensor id
+    uint64_t base = 0;        // dither index of its element 0 within the descriptor
     int kind = 0, momentum = 0, decay = 0, vec = 0;
     int64_t n = 0, m = 0, numel = 0;
     int64_t moff = -1, voff = -1, roff = -1, coff = -1;  // floats into the state
@@ -43,7 +48,8 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 struct skew_handle {
     std::vector<skew_param_desc_t> desc;
     skew_hparams_t hp{};
-    std::vector<TPlan> t;
+    std::vector<TPlan> t;                  // matrices / vectors in descriptor order
+    std::vector<uint32_t> first, count;    // per descriptor: its first plan and how many
     size_t state_bytes = 0, ws_bytes = 0;
     size_t ws_scal = 0, ws_fb = 0, ws_err = 0, ws_tab = 0, ws_tab_end = 0;
     size_t ws_tens = 0, ws_itemsA = 0, ws_itemsR = 0, ws_itemsF = 0, ws_itemsB = 0, ws_itemsC = 0, ws_itemsCR = 0;
@@ -139,7 +145,8 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     try {
         h->hp = H;
         h->desc.assign(params, params + n_params);
-        h->t.resize(n_params);
+        h->first.assign(n_params, 0);
+        h->count.assign(n_params, 0);
     } catch (...) {
         delete h;
         return fail(nullptr, SKEW_ENOMEM, "out of host memory");
@@ -147,26 +154,43 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     const int64_t kMaxExtent = int64_t(1) << 40;
     for (int32_t k = 0; k < n_params; ++k) {
         const skew_param_desc_t &d = params[k];
-        TPlan &p = h->t[k];
+        TPlan p;
         if (!d.weight || !d.grad) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: null weight or grad", k); }
         if (((uintptr_t)d.weight & 1) || ((uintptr_t)d.grad & 1)) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: bf16 pointers must be 2-byte aligned", k); }
-        if (d.ndim != 1 && d.ndim != 2) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: ndim must be 1 or 2", k); }
+        if (d.ndim < 1 || d.ndim > 3) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: ndim must be 1, 2 or 3", k); }
         if (d.tier < SKEW_TIER_BACKBONE || d.tier > SKEW_TIER_ROUTER) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: unknown tier %d", k, d.tier); }
         if (d.flags & ~SKEW_F_NO_DECAY) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: unknown flags", k); }
-        if (d.reserved != 0) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: reserved must be 0", k); }
+        if (d.ndim == 3 ? d.stack < 1 : d.stack != 0) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: stack must be >= 1 when ndim == 3 and 0 otherwise", k); }
+        const int64_t E = d.ndim == 3 ? (int64_t)d.stack : 1;
         p.n = d.shape[0];
-        p.m = d.ndim == 2 ? d.shape[1] : 1;
+        p.m = d.ndim >= 2 ? d.shape[1] : 1;
         if (p.n < 1 || p.m < 1 || p.n > kMaxExtent || p.m > kMaxExtent) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: extents must be in [1, 2^40]", k); }
-        if (p.n > (int64_t(1) << 62) / p.m) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: too many elements", k); }
+        if (p.n > (int64_t(1) << 62) / p.m || p.n * p.m > (int64_t(1) << 62) / E) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: too many elements", k); }
         p.numel = p.n * p.m;
-        resolve(d.ndim, d.tier, H.policy, d.flags, p);
-        // tiles are indexed with 32 bits: at most 2^31 per tensor
+        resolve(d.ndim == 3 ? 2 : d.ndim, d.tier, H.policy, d.flags, p);  // every matrix of a stack is a matrix
+        // tiles are indexed with 32 bits: at most 2^31 per matrix
         const int64_t tiles64 = p.kind == kKindFactored ? ((p.m + 255) / 256) * ((p.n + 255) / 256)
                                                         : (p.numel + kFlatTileElems - 1) / kFlatTileElems;
         if (tiles64 > (int64_t(1) << 31)) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: too many elements", k); }
-        geometry(p, (((uintptr_t)d.weight | (uintptr_t)d.grad) & 15) == 0);
-        h->n_rowpath += p.rowpath;
+        try {
+            h->first[k] = (uint32_t)h->t.size();
+            h->count[k] = (uint32_t)E;
+            for (int64_t e = 0; e < E; ++e) {
+                TPlan q = p;
+                q.w = (uint16_t *)d.weight + e * p.numel;
+                q.g = (const uint16_t *)d.grad + e * p.numel;
+                q.tid = (uint32_t)k;
+                q.base = (uint64_t)(e * p.numel);
+                geometry(q, (((uintptr_t)q.w | (uintptr_t)q.g) & 15) == 0);
+                h->n_rowpath += q.rowpath;
+                h->t.push_back(q);
+            }
+        } catch (...) {
+            delete h;
+            return fail(nullptr, SKEW_ENOMEM, "out of host memory");
+        }
     }
+    const int32_t n_plans = (int32_t)h->t.size();
 
     // State layout (fp32 offsets): [momentum arrays][full v arrays][R arrays][C arrays].
     // Arrays whose length is a multiple of 4 come first in each group so that as
@@ -187,7 +211,7 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     // Item tables: every factored tensor's tiles (phase A), finalize items
     // (phase F) and every tensor's tiles (phases B and C), tensors in order.
     try {
-        for (int q = 0; q < n_params; ++q) {
+        for (int q = 0; q < n_plans; ++q) {
             const TPlan &p = h->t[q];
             if (p.kind == kKindFactored) {
                 if (p.rowpath)
@@ -212,14 +236,14 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     // path's phase-B queue ([count][tensor ids]) are zeroed every step.
     size_t w = 0;
     h->ws_scal = w;
-    w = align_up(w + sizeof(TensorScal) * n_params, 256);
+    w = align_up(w + sizeof(TensorScal) * n_plans, 256);
     h->ws_fb = w;
     w = align_up(w + 4 * (size_t(h->n_rowpath) + 1), 256);
     h->ws_err = w;
     w = align_up(w + 16, 256);
     h->ws_tab = w;
     h->ws_tens = w;
-    w = align_up(w + sizeof(TensorDev) * n_params, 256);
+    w = align_up(w + sizeof(TensorDev) * n_plans, 256);
     auto table = [&](size_t &at, const std::vector<uint2> &v) {
         at = w;
         w = align_up(w + sizeof(uint2) * v.size(), 256);
@@ -263,7 +287,7 @@ size_t skew_state_bytes(const skew_handle_t *h) { return h ? h->state_bytes : 0;
 
 size_t skew_workspace_bytes(const skew_handle_t *h) { return h ? h->ws_bytes : 0; }
 
-int32_t skew_num_tensors(const skew_handle_t *h) { return h ? (int32_t)h->t.size() : 0; }
+int32_t skew_num_tensors(const skew_handle_t *h) { return h ? (int32_t)h->desc.size() : 0; }
 
 int64_t skew_launches_per_step(const skew_handle_t *h) {
     if (!h) return 0;
@@ -276,21 +300,21 @@ const char *skew_last_error(const skew_handle_t *h) { return h ? h->err.c_str() 
 
 int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *out) {
     if (!h || !out) return SKEW_EINVAL;
-    if (tid < 0 || tid >= (int32_t)h->t.size()) return fail(const_cast<skew_handle_t *>(h), SKEW_EINVAL, "tid %d out of range", tid);
-    const TPlan &p = h->t[tid];
+    if (tid < 0 || tid >= (int32_t)h->desc.size()) return fail(const_cast<skew_handle_t *>(h), SKEW_EINVAL, "tid %d out of range", tid);
+    const TPlan &p = h->t[h->first[tid]];  // a stack's matrices share kind, shape and path; arrays follow on
     out->kind = p.kind;
     out->momentum = p.momentum;
     out->decay = p.decay;
     out->vectorized = p.vec;
     out->rows = p.n;
     out->cols = p.m;
-    out->numel = p.numel;
+    out->numel = p.numel * (int64_t)h->count[tid];
     out->m_offset = p.moff;
     out->v_offset = p.voff;
     out->r_offset = p.roff;
     out->c_offset = p.coff;
     out->rowpath = (int32_t)p.rowpath;
-    out->reserved = 0;
+    out->stack = h->desc[tid].ndim == 3 ? (int32_t)h->count[tid] : 0;
     return SKEW_OK;
 }
 
@@ -317,10 +341,9 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
     auto al16 = [](const void *p) { return ((uintptr_t)p & 15) == 0; };
     for (size_t k = 0; k < h->t.size(); ++k) {
         TPlan &p = h->t[k];
-        const skew_param_desc_t &d = h->desc[k];
         TensorDev &T = td[k];
-        T.w = (uint16_t *)d.weight;
-        T.g = (const uint16_t *)d.grad;
+        T.w = (uint16_t *)p.w;
+        T.g = (const uint16_t *)p.g;
         T.M = p.moff >= 0 ? sf + p.moff : nullptr;
         T.v = p.voff >= 0 ? sf + p.voff : nullptr;
         T.R = p.roff >= 0 ? sf + p.roff : nullptr;
@@ -338,7 +361,8 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.n = p.n;
         T.m = p.m;
         T.numel = p.numel;
-        T.tid = (uint32_t)k;
+        T.tid = p.tid;
+        T.base = p.base;
         T.kind = p.kind;
         T.momentum = p.momentum;
         T.decay = p.decay;
@@ -510,14 +534,20 @@ int skew_sync_status(skew_handle_t *h, void *stream) {
 }
 
 int skew_tensor_scalars(skew_handle_t *h, int32_t tid, double out[4], void *stream) {
+    return skew_matrix_scalars(h, tid, 0, out, stream);
+}
+
+int skew_matrix_scalars(skew_handle_t *h, int32_t tid, int32_t e, double out[4], void *stream) {
     if (!h || !out) return SKEW_EINVAL;
-    if (tid < 0 || tid >= (int32_t)h->t.size()) return fail(h, SKEW_EINVAL, "tid %d out of range", tid);
+    if (tid < 0 || tid >= (int32_t)h->desc.size()) return fail(h, SKEW_EINVAL, "tid %d out of range", tid);
+    if (e < 0 || e >= (int32_t)h->count[tid]) return fail(h, SKEW_EINVAL, "matrix %d of tensor %d out of range", e, tid);
     if (!h->bound) return fail(h, SKEW_ESTATE, "not bound");
-    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
-    if (e != cudaSuccess) return cuda_fail(h, e, "stream synchronize");
+    const size_t k = h->first[tid] + (uint32_t)e;
+    cudaError_t err = cudaStreamSynchronize((cudaStream_t)stream);
+    if (err != cudaSuccess) return cuda_fail(h, err, "stream synchronize");
     TensorScal sc;
-    e = cudaMemcpy(&sc, h->ws + h->ws_scal + sizeof(TensorScal) * tid, sizeof sc, cudaMemcpyDeviceToHost);
-    if (e != cudaSuccess) return cuda_fail(h, e, "scalar read");
+    err = cudaMemcpy(&sc, h->ws + h->ws_scal + sizeof(TensorScal) * k, sizeof sc, cudaMemcpyDeviceToHost);
+    if (err != cudaSuccess) return cuda_fail(h, err, "scalar read");
     out[0] = sc.rbar;
     out[1] = sc.sumsq;
     out[2] = sc.rms;

@@ -156,15 +156,18 @@ __device__ __forceinline__ uint4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_
 // the two halves of the seed (kept in registers by the hot loops).
 struct Dith {
     uint32_t tid, step, k0, k1;
+    uint64_t base;  // dither index of the tile's tensor element 0
 };
 
-__device__ __forceinline__ Dith dith_of(const StepArgs &A, uint32_t tid) { return Dith{tid, A.step_lo, A.seed_lo, A.seed_hi}; }
+__device__ __forceinline__ Dith dith_of(const StepArgs &A, const TensorDev &T) {
+    return Dith{T.tid, A.step_lo, A.seed_lo, A.seed_hi, T.base};
+}
 
 // The 16-bit dithers of the eight elements idx0 .. idx0+7 (idx0 a multiple of 8):
 // counter (idx0/8 lo, idx0/8 hi, tensor id, step lo), key (seed lo, seed hi);
 // element k takes half (k & 1) of word k >> 1.
 __device__ __forceinline__ void dither8(uint64_t idx0, const Dith &d, uint32_t (&r)[8]) {
-    const uint64_t blk = idx0 >> 3;
+    const uint64_t blk = (idx0 + d.base) >> 3;
     const uint4 o = philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), d.tid, d.step, d.k0, d.k1);
     const uint32_t w[4] = {o.x, o.y, o.z, o.w};
 #pragma unroll
@@ -175,6 +178,7 @@ __device__ __forceinline__ void dither8(uint64_t idx0, const Dith &d, uint32_t (
 }
 
 __device__ __forceinline__ uint32_t dither1(uint64_t idx, const Dith &d) {
+    idx += d.base;
     const uint64_t blk = idx >> 3;
     const uint4 o = philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), d.tid, d.step, d.k0, d.k1);
     const uint32_t k = (uint32_t)(idx & 7);
@@ -1174,7 +1178,7 @@ __device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const Ten
     uint16_t *__restrict__ w_ = T.w;
     const int64_t n = T.n, m = T.m, row0 = F.row0, RG = F.RG, col0 = F.col0;
     const int valid = F.valid;
-    const Dith d = dith_of(A, T.tid);
+    const Dith d = dith_of(A, T);
     const float coefC = __ldcg(&S.coefC);
     const float wdf = T.decay ? A.wdf : 1.0f;
     const float ce = A.ce;
@@ -1249,7 +1253,7 @@ __device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const Ten
             const float a = rows[k * RG];
 #pragma unroll
             for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], ce), w[c] * wdf);
-            write8<false>(w_, d, e0, valid, (e0 & 7) == 0, x, pol);
+            write8<false>(w_, d, e0, valid, ((e0 + d.base) & 7) == 0, x, pol);
         }
     }
 }
@@ -1277,7 +1281,8 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
             load_bf8_scalar(T.w + e0, valid, w);
 #pragma unroll
         for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(__frsqrt_rn(v[c]), A.ce), w[c] * wdf);
-        write8<VEC>(T.w, dith_of(A, T.tid), e0, valid, true, x, pol);
+        const Dith dd = dith_of(A, T);  // on the vector path e0 and base are multiples of 8
+        write8<VEC>(T.w, dd, e0, valid, VEC || ((e0 + dd.base) & 7) == 0, x, pol);
     }
 }
 
@@ -1319,7 +1324,7 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
     const int tid = threadIdx.x;
     const int64_t m = 8 * V;
     uint16_t *__restrict__ w_ = T.w;
-    const Dith d = dith_of(A, T.tid);
+    const Dith d = dith_of(A, T);
     const float wdf = T.decay ? A.wdf : 1.0f;
     const float ce = A.ce;
     const float2 wdf2 = make_float2(wdf, wdf);

@@ -87,6 +87,7 @@ struct TensorDev {
     float2 *u2;         // per tile sum of (U / coef)^2 as a (hi, lo) pair [ntiles]
     int64_t n, m, numel;
     uint32_t tid;       // dither tensor id
+    uint64_t base;      // dither index of element 0 (a matrix of a stacked tensor: its offset)
     uint32_t kind, momentum, decay;
     uint32_t vec;       // 1: 16-byte vector loads / stores are legal
     uint32_t lcl;       // factored: log2 of lanes along a row (LC)

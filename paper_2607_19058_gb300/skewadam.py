@@ -26,7 +26,7 @@ F_NO_DECAY = 1
 KIND_FULL, KIND_FACTORED = 0, 1
 
 EXPORTS = ["skew_create", "skew_destroy", "skew_state_bytes", "skew_workspace_bytes", "skew_bind", "skew_step",
-           "skew_sync_status", "skew_tensor_scalars", "skew_tensor_info", "skew_num_tensors", "skew_last_error",
+           "skew_sync_status", "skew_tensor_scalars", "skew_matrix_scalars", "skew_tensor_info", "skew_num_tensors", "skew_last_error",
            "skew_profile_begin", "skew_profile_end", "skew_kernel_name", "skew_step_tensor_noalloc",
            "skew_launches_per_step"]
 
@@ -39,7 +39,7 @@ class SkewError(RuntimeError):
 
 class ParamDesc(C.Structure):
     _fields_ = [("weight", C.c_void_p), ("grad", C.c_void_p), ("shape", C.c_int64 * 2), ("ndim", C.c_int32),
-                ("tier", C.c_int32), ("flags", C.c_uint32), ("reserved", C.c_uint32)]
+                ("tier", C.c_int32), ("flags", C.c_uint32), ("stack", C.c_uint32)]
 
 
 class HParams(C.Structure):
@@ -51,7 +51,7 @@ class TensorInfo(C.Structure):
     _fields_ = [("kind", C.c_int32), ("momentum", C.c_int32), ("decay", C.c_int32), ("vectorized", C.c_int32),
                 ("rows", C.c_int64), ("cols", C.c_int64), ("numel", C.c_int64), ("m_offset", C.c_int64),
                 ("v_offset", C.c_int64), ("r_offset", C.c_int64), ("c_offset", C.c_int64), ("rowpath", C.c_int32),
-                ("reserved", C.c_int32)]
+                ("stack", C.c_int32)]
 
 
 _lock = threading.Lock()
@@ -86,6 +86,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
         L.skew_sync_status.restype = C.c_int
         L.skew_tensor_scalars.argtypes = [vp, i32, C.POINTER(C.c_double), vp]
         L.skew_tensor_scalars.restype = C.c_int
+        L.skew_matrix_scalars.argtypes = [vp, i32, i32, C.POINTER(C.c_double), vp]
+        L.skew_matrix_scalars.restype = C.c_int
         L.skew_tensor_info.argtypes = [vp, i32, C.POINTER(TensorInfo)]
         L.skew_tensor_info.restype = C.c_int
         L.skew_launches_per_step.argtypes = [vp]
@@ -154,6 +156,12 @@ def skew_tensor_scalars(h, tid: int, stream: int):
     return {"rbar": out[0], "sumu2": out[1], "rms": out[2], "kappa": out[3]}
 
 
+def skew_matrix_scalars(h, tid: int, e: int, stream: int):
+    out = (C.c_double * 4)()
+    _check(load().skew_matrix_scalars(h, tid, e, out, stream), h)
+    return {"rbar": out[0], "sumu2": out[1], "rms": out[2], "kappa": out[3]}
+
+
 def skew_tensor_info(h, tid: int) -> TensorInfo:
     info = TensorInfo()
     _check(load().skew_tensor_info(h, tid, C.byref(info)), h)
@@ -214,8 +222,10 @@ def hparams(beta1=0.9, beta2=0.999, eps=1e-8, clip_d=1.0, weight_decay=0.05, pol
 class SkewAdam:
     """SkewAdam over a list of (weight, grad, tier[, flags]) bf16 CUDA tensors.
 
-    The optimizer state is one device buffer of exactly ``state_bytes`` bytes
-    (the paper's closed form); the workspace holds scratch and tables.
+    A 3-D tensor (E, n, m) is a stack of E matrices (e.g. an MoE layer's experts
+    kept in one array), each stepped with its own second-moment factors and clip
+    factor. The optimizer state is one device buffer of exactly ``state_bytes``
+    bytes (the paper's closed form); the workspace holds scratch and tables.
     """
 
     def __init__(self, params: Iterable, hp: HParams, stream=None):
@@ -230,10 +240,13 @@ class SkewAdam:
                 raise TypeError("weights and gradients must be bf16")
             if not (w.is_cuda and g.is_cuda and w.is_contiguous() and g.is_contiguous()):
                 raise ValueError("weights and gradients must be contiguous CUDA tensors")
-            if w.shape != g.shape or w.dim() not in (1, 2):
-                raise ValueError("weight / grad shapes must match and be 1-D or 2-D")
-            shape = (int(w.shape[0]), int(w.shape[1]) if w.dim() == 2 else 0)
-            descs.append(ParamDesc(w.data_ptr(), g.data_ptr(), (C.c_int64 * 2)(*shape), w.dim(), tier, flags, 0))
+            if w.shape != g.shape or w.dim() not in (1, 2, 3):
+                raise ValueError("weight / grad shapes must match and be 1-D, 2-D or 3-D")
+            if w.dim() == 3:
+                shape, stack = (int(w.shape[1]), int(w.shape[2])), int(w.shape[0])
+            else:
+                shape, stack = (int(w.shape[0]), int(w.shape[1]) if w.dim() == 2 else 0), 0
+            descs.append(ParamDesc(w.data_ptr(), g.data_ptr(), (C.c_int64 * 2)(*shape), w.dim(), tier, flags, stack))
             self.params.append((w, g))
         self.hp = hp
         self.h = skew_create(descs, hp)
@@ -262,8 +275,10 @@ class SkewAdam:
     def sync_status(self, stream=None) -> None:
         skew_sync_status(self.h, self._stream(stream))
 
-    def scalars(self, tid: int, stream=None):
-        return skew_tensor_scalars(self.h, tid, self._stream(stream))
+    def scalars(self, tid: int, stream=None, matrix: int = 0):
+        """mean(R), sum of U^2, RMS and clip factor of tensor `tid` (of its matrix
+        `matrix` when it is a stack)."""
+        return skew_matrix_scalars(self.h, tid, matrix, self._stream(stream))
 
     def info(self, tid: int) -> TensorInfo:
         return skew_tensor_info(self.h, tid)
@@ -273,8 +288,9 @@ class SkewAdam:
         f = self.state[: self.state_bytes].view(self.torch.float32)
         i = self.info(tid)
         out = {}
-        for key, off, cnt in (("M", i.m_offset, i.numel), ("v", i.v_offset, i.numel), ("R", i.r_offset, i.rows),
-                              ("C", i.c_offset, i.cols)):
+        E = max(1, i.stack)  # a stack's arrays hold its matrices' in order
+        for key, off, cnt in (("M", i.m_offset, i.numel), ("v", i.v_offset, i.numel), ("R", i.r_offset, E * i.rows),
+                              ("C", i.c_offset, E * i.cols)):
             out[key] = None if off < 0 else f[off: off + cnt]
         return out
 

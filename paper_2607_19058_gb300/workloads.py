@@ -165,6 +165,22 @@ def small() -> Workload:
     return Workload("small", specs, HP(), "normal", steps=20, n_experts=32)
 
 
+def stack_experts(wl: Workload) -> Workload:
+    """The same parameter set with each expert weight kept as one (E, n, m) array
+    over the experts (how MoE layers usually store them); other tensors as they are."""
+    shapes, rest, first = {}, [], None
+    for k, s in enumerate(wl.specs):
+        if s.tier == TIER_EXPERT and s.expert >= 0:
+            slot = s.name.rsplit(".", 1)[1]
+            shapes.setdefault(slot, (s.shape, []))[1].append(s.expert)
+            first = len(rest) if first is None else first
+        else:
+            rest.append(s)
+    stacks = [Spec(f"experts.{slot}", (len(es),) + tuple(shp), TIER_EXPERT) for slot, (shp, es) in shapes.items()]
+    specs = rest[:first] + stacks + rest[first:] if stacks else rest
+    return dataclasses.replace(wl, name=wl.name + "_stacked", specs=specs, grad_kind="normal")
+
+
 WORKLOADS = {"small": small, "toy": toy, "slice": slice_, "appb": appb, "literal": literal, "skewed": skewed,
              "ablation": ablation}
 

@@ -21,7 +21,9 @@ post-step results are compared with the acceptance bars of the method:
     draw r or a wrong update is not admitted by the bound;
   * per-tensor RMS(U) and clip factor: relative error <= 1e-6.
 Tensors are independent, so checking a subset of a large parameter set is
-exact parity for that subset while the GPU runs the whole set.
+exact parity for that subset while the GPU runs the whole set. A stacked
+(E, n, m) tensor is checked as E matrices, each against its own oracle run
+whose dither index starts at the matrix's flat offset e*n*m.
 """
 from __future__ import annotations
 
@@ -144,7 +146,8 @@ class Harness:
 
     def __init__(self, wl: WL.Workload, check: Optional[Sequence[int]] = None, device="cuda",
                  grad_device: Optional[str] = None, hp_override: Optional[dict] = None,
-                 misalign: Sequence[int] = ()):
+                 misalign: Sequence[int] = (), matrices: Optional[Dict[int, Sequence[int]]] = None):
+        """`matrices[k]`, when given, limits the check of stacked tensor k to those matrices."""
         self.wl = wl
         hpd = dataclasses.asdict(wl.hp)
         if hp_override:
@@ -170,8 +173,8 @@ class Harness:
         self.hp = S.hparams(hpd["beta1"], hpd["beta2"], hpd["eps"], hpd["clip_d"], hpd["weight_decay"], hpd["policy"])
         self.opt = S.SkewAdam(params, self.hp)
         self.check = list(range(len(wl.specs))) if check is None else list(check)
-        self.ostate = {k: O.TensorState(wl.specs[k].shape, wl.specs[k].tier, hpd["policy"], wl.specs[k].no_decay)
-                       for k in self.check}
+        self.ostate = {k: {e: O.TensorState(self._mat_shape(k), wl.specs[k].tier, hpd["policy"], wl.specs[k].no_decay)
+                           for e in (matrices or {}).get(k, range(self._stack(k)))} for k in self.check}
         self.ohp = O.hparams(hpd["beta1"], hpd["beta2"], hpd["eps"], hpd["clip_d"], hpd["weight_decay"])
         self.lr = hpd["lr"]
 
@@ -179,9 +182,25 @@ class Harness:
         for k in range(len(self.wl.specs)):
             self.G[k].copy_(WL.grad(self.wl, k, t, self.gdev).to(self.dev))
 
-    def _gpu_state(self, k: int) -> Dict[str, Optional[np.ndarray]]:
-        v = self.opt.state_views(k)
-        return {key: (None if a is None else f32(a)) for key, a in v.items()}
+    def _stack(self, k: int) -> int:
+        return self.wl.specs[k].shape[0] if len(self.wl.specs[k].shape) == 3 else 1
+
+    def _mat_shape(self, k: int):
+        shp = self.wl.specs[k].shape
+        return tuple(shp[1:]) if len(shp) == 3 else tuple(shp)
+
+    def _gpu_state(self, k: int) -> List[Dict[str, Optional[np.ndarray]]]:
+        """Per matrix of tensor k (one entry unless it is a stack): its M, v, R, C."""
+        v = {key: (None if a is None else f32(a)) for key, a in self.opt.state_views(k).items()}
+        E = self._stack(k)
+        out = []
+        for e in range(E):
+            d = {}
+            for key, a in v.items():
+                ln = None if a is None else a.size // E
+                d[key] = None if a is None else a[e * ln:(e + 1) * ln]
+            out.append(d)
+        return out
 
     def step(self, t: int, seed: int = 1234, grads_loaded: bool = False) -> Report:
         if not grads_loaded:
@@ -189,53 +208,61 @@ class Harness:
         torch.cuda.synchronize()
         pre = {}
         for k in self.check:   # teacher forcing: the oracle starts from the GPU's pre-step values
-            st = self.ostate[k]
             gs = self._gpu_state(k)
-            for key in ("M", "v", "R", "C"):
-                if getattr(st, key) is not None:
-                    getattr(st, key)[:] = gs[key]
-            pre[k] = (bits16(self.W[k]), bits16(self.G[k]), None if st.M is None else st.M.copy())
+            wb, gb = bits16(self.W[k]), bits16(self.G[k])
+            nm = wb.size // self._stack(k)
+            pre[k] = {}
+            for e, st in self.ostate[k].items():
+                for key in ("M", "v", "R", "C"):
+                    if getattr(st, key) is not None:
+                        getattr(st, key)[:] = gs[e][key]
+                pre[k][e] = (wb[e * nm:(e + 1) * nm].copy(), gb[e * nm:(e + 1) * nm].copy(),
+                             None if st.M is None else st.M.copy())
         self.opt.step(t, self.lr, seed)
         self.opt.sync_status()
         rep = Report()
         for k in self.check:
-            w0, g, m_prev = pre[k]
-            wpre = w0.copy()
-            st = self.ostate[k]
-            o = O.tensor_step(w0, g, st, k, self.ohp, t, self.lr, seed, want_x=True)
-            where = f"{self.wl.name}/{self.wl.specs[k].name} step {t}"
-            gw = bits16(self.W[k])
-            lam = float(np.float32(self.hpd["weight_decay"])) if st.decay else 0.0
-            wdf = 1.0 - float(np.float32(self.lr)) * lam
-            terms = self._momentum_update_terms(st, o, g, m_prev, t) if st.momentum else None
-            nbad, worst = compare_weights(gw, w0, o["x"], o["r"], wpre, wdf, where, terms)
-            gs = self._gpu_state(k)
-            worst_state = 0.0
-            for key in ("M", "v", "R", "C"):
-                if getattr(st, key) is not None:
-                    if key == "M":
-                        gd = (g.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
-                        b1 = float(np.float32(self.hpd["beta1"]))
-                        scale = b1 * np.abs(m_prev.astype(np.float64)) + (1 - b1) * np.abs(gd)
-                        e = rel_err_terms(gs[key], st.M, scale)
-                    else:
-                        e = rel_err(gs[key], getattr(st, key))
-                    assert e <= STATE_RTOL, f"{where}: state {key} rel err {e:.3g}"
-                    worst_state = max(worst_state, e)
-            sc = self.opt.scalars(k)
-            se = 0.0
-            for key in ("rms", "kappa"):
-                e = abs(sc[key] - o[key]) / max(abs(o[key]), 1e-300)
-                if o[key] == 0.0:
-                    e = abs(sc[key])
-                assert e <= SCALAR_RTOL, f"{where}: {key} {sc[key]!r} vs oracle {o[key]!r}"
-                se = max(se, e)
-            r = Report(elements=gw.size, w_mismatch=nbad, worst_state_rel=worst_state, worst_scalar_rel=se,
-                       worst_thresh=worst, clipped=int(o["kappa"] < 1.0), tensors=1)
-            rep.merge(r)
+            gws, gss = bits16(self.W[k]), self._gpu_state(k)
+            for e, st in self.ostate[k].items():
+                rep.merge(self._check_matrix(k, e, st, pre[k][e], gws, gss[e], t, seed))
         assert rep.w_mismatch <= W_MISMATCH_FRAC * rep.elements, \
             f"{self.wl.name} step {t}: {rep.w_mismatch} of {rep.elements} weights differ"
         return rep
+
+    def _check_matrix(self, k, e, st, pre, gws, gs, t, seed) -> Report:
+        """Matrix e of tensor k (e = 0 unless it is a stack) against one oracle step."""
+        w0, g, m_prev = pre
+        wpre = w0.copy()
+        nm = w0.size
+        o = O.tensor_step(w0, g, st, k, self.ohp, t, self.lr, seed, want_x=True, idx0=e * nm)
+        where = f"{self.wl.name}/{self.wl.specs[k].name}" + (f"[{e}]" if self._stack(k) > 1 else "") + f" step {t}"
+        gw = gws[e * nm:(e + 1) * nm]
+        lam = float(np.float32(self.hpd["weight_decay"])) if st.decay else 0.0
+        wdf = 1.0 - float(np.float32(self.lr)) * lam
+        terms = self._momentum_update_terms(st, o, g, m_prev, t) if st.momentum else None
+        nbad, worst = compare_weights(gw, w0, o["x"], o["r"], wpre, wdf, where, terms)
+        worst_state = 0.0
+        for key in ("M", "v", "R", "C"):
+            if getattr(st, key) is not None:
+                if key == "M":
+                    gd = (g.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+                    b1 = float(np.float32(self.hpd["beta1"]))
+                    scale = b1 * np.abs(m_prev.astype(np.float64)) + (1 - b1) * np.abs(gd)
+                    err = rel_err_terms(gs[key], st.M, scale)
+                else:
+                    err = rel_err(gs[key], getattr(st, key))
+                assert err <= STATE_RTOL, f"{where}: state {key} rel err {err:.3g}"
+                worst_state = max(worst_state, err)
+        sc = self.opt.scalars(k, matrix=e)
+        se = 0.0
+        for key in ("rms", "kappa"):
+            err = abs(sc[key] - o[key]) / max(abs(o[key]), 1e-300)
+            if o[key] == 0.0:
+                err = abs(sc[key])
+            assert err <= SCALAR_RTOL, f"{where}: {key} {sc[key]!r} vs oracle {o[key]!r}"
+            se = max(se, err)
+        return Report(elements=gw.size, w_mismatch=nbad, worst_state_rel=worst_state, worst_scalar_rel=se,
+                      worst_thresh=worst, clipped=int(o["kappa"] < 1.0), tensors=1)
 
     def _momentum_update_terms(self, st, o, g, m_prev, t):
         """lr*kappa*coef/D * (b1|M_prev| + (1-b1)|g|) from the oracle's post-step state."""

@@ -51,9 +51,10 @@ def test_struct_layout_matches_header():
     #include <stddef.h>
     #include "skewadam.h"
     int main(void) {
-      printf("%zu %zu %zu %zu %zu %zu %zu\n", sizeof(skew_param_desc_t), sizeof(skew_hparams_t),
+      printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(skew_param_desc_t), sizeof(skew_hparams_t),
              sizeof(skew_tensor_info_t), offsetof(skew_param_desc_t, shape), offsetof(skew_param_desc_t, ndim),
-             offsetof(skew_param_desc_t, flags), offsetof(skew_tensor_info_t, m_offset));
+             offsetof(skew_param_desc_t, flags), offsetof(skew_tensor_info_t, m_offset),
+             offsetof(skew_param_desc_t, stack), offsetof(skew_tensor_info_t, stack));
       return 0; }
     '''
     with tempfile.TemporaryDirectory() as d:
@@ -62,16 +63,17 @@ def test_struct_layout_matches_header():
         subprocess.check_call(["gcc", "-I", os.path.dirname(HEADER), src, "-o", exe])
         got = [int(x) for x in subprocess.check_output([exe]).split()]
     want = [C.sizeof(S.ParamDesc), C.sizeof(S.HParams), C.sizeof(S.TensorInfo), S.ParamDesc.shape.offset,
-            S.ParamDesc.ndim.offset, S.ParamDesc.flags.offset, S.TensorInfo.m_offset.offset]
+            S.ParamDesc.ndim.offset, S.ParamDesc.flags.offset, S.TensorInfo.m_offset.offset,
+            S.ParamDesc.stack.offset, S.TensorInfo.stack.offset]
     assert got == want
 
 
 def _descs(wl, base=0x100000):
     out = []
     for k, s in enumerate(wl.specs):
-        shp = (s.shape[0], s.shape[1] if len(s.shape) == 2 else 0)
+        shp = tuple(s.shape[1:]) if len(s.shape) == 3 else (s.shape[0], s.shape[1] if len(s.shape) == 2 else 0)
         out.append(S.ParamDesc(base * (k + 1), base * (k + 1) + 64, (C.c_int64 * 2)(*shp), len(s.shape), s.tier,
-                               S.F_NO_DECAY if s.no_decay else 0, 0))
+                               S.F_NO_DECAY if s.no_decay else 0, s.shape[0] if len(s.shape) == 3 else 0))
     return out
 
 
@@ -88,6 +90,47 @@ def test_state_bytes_is_closed_form(name):
 def test_appb_headline_state_bytes():
     h = S.skew_create(_descs(WL.appb()), S.hparams())
     assert S.skew_state_bytes(h) == 1_380_800_000
+    S.skew_destroy(h)
+
+
+@pytest.mark.parametrize("name", ["toy", "appb", "ablation"])
+def test_stacked_experts_plan_like_separate_matrices(name):
+    """Experts kept as (E, n, m) stacks: each matrix keeps its own factors, so the state
+    is the closed form of the E separate matrices; a stack's arrays are contiguous."""
+    wl, st = WL.get(name), WL.stack_experts(WL.get(name))
+    assert any(len(s.shape) == 3 for s in st.specs)
+    for policy in (wl.hp.policy, S.POLICY_UNIFORM):
+        h = S.skew_create(_descs(st), S.hparams(policy=policy))
+        want = O.state_bytes([(s.shape, s.tier) for s in wl.specs], policy)
+        assert S.skew_state_bytes(h) == want
+        assert S.skew_num_tensors(h) == len(st.specs)
+        total = S.skew_state_bytes(h) // 4
+        spans = []
+        for k, s in enumerate(st.specs):
+            i = S.skew_tensor_info(h, k)
+            E = s.shape[0] if len(s.shape) == 3 else 1
+            assert i.stack == (E if len(s.shape) == 3 else 0)
+            assert (i.rows, i.cols) == ((s.shape[-2], s.shape[-1]) if len(s.shape) >= 2 else (s.shape[0], 1))
+            assert i.numel == s.numel
+            for off, cnt in ((i.m_offset, i.numel), (i.v_offset, i.numel), (i.r_offset, E * i.rows),
+                             (i.c_offset, E * i.cols)):
+                if off >= 0:
+                    spans.append((off, off + cnt))
+        spans.sort()
+        assert spans[0][0] == 0 and spans[-1][1] == total
+        assert all(a[1] == b[0] for a, b in zip(spans, spans[1:]))
+        S.skew_destroy(h)
+
+
+def test_matrix_scalars_range():
+    h = S.skew_create([_one((3, 4, 8)), _one((4, 8))], S.hparams())
+    for tid, e in ((0, 3), (0, -1), (1, 1), (2, 0)):
+        with pytest.raises(S.SkewError) as err:
+            S.skew_matrix_scalars(h, tid, e, 0)
+        assert err.value.code == S.SKEW_EINVAL
+    with pytest.raises(S.SkewError) as err:   # in range, but nothing is bound yet
+        S.skew_matrix_scalars(h, 0, 2, 0)
+    assert err.value.code == S.SKEW_ESTATE
     S.skew_destroy(h)
 
 
@@ -116,15 +159,16 @@ def test_state_layout_tiles_the_buffer(name):
 
 
 def _one(shape=(4, 8), tier=S.TIER_EXPERT, **kw):
-    d = dict(weight=0x1000, grad=0x2000, ndim=len(shape), tier=tier, flags=0, reserved=0)
+    d = dict(weight=0x1000, grad=0x2000, ndim=len(shape), tier=tier, flags=0, stack=shape[0] if len(shape) == 3 else 0)
     d.update(kw)
-    shp = (shape[0], shape[1] if len(shape) == 2 else 0)
-    return S.ParamDesc(d["weight"], d["grad"], (C.c_int64 * 2)(*shp), d["ndim"], d["tier"], d["flags"], d["reserved"])
+    shp = tuple(shape[-2:]) if len(shape) == 3 else (shape[0], shape[1] if len(shape) == 2 else 0)
+    return S.ParamDesc(d["weight"], d["grad"], (C.c_int64 * 2)(*shp), d["ndim"], d["tier"], d["flags"], d["stack"])
 
 
 @pytest.mark.parametrize("desc,msg", [
-    (dict(weight=0), "null"), (dict(grad=0), "null"), (dict(weight=0x1001), "aligned"), (dict(ndim=3), "ndim"),
-    (dict(tier=5), "tier"), (dict(flags=8), "flags"), (dict(reserved=1), "reserved"),
+    (dict(weight=0), "null"), (dict(grad=0), "null"), (dict(weight=0x1001), "aligned"), (dict(ndim=4), "ndim"),
+    (dict(ndim=0), "ndim"), (dict(tier=5), "tier"), (dict(flags=8), "flags"), (dict(stack=1), "stack"),
+    (dict(ndim=3, stack=0), "stack"),
 ])
 def test_create_rejects_bad_descriptors(desc, msg):
     with pytest.raises(S.SkewError) as e:

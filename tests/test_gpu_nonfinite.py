@@ -75,8 +75,8 @@ def test_nonfinite_gradients_follow_the_oracle():
         torch.cuda.synchronize()
         pre = {}
         for k in range(len(specs)):  # teacher forcing from the GPU's pre-step state
-            st = h.ostate[k]
-            gs = h._gpu_state(k)
+            st = h.ostate[k][0]
+            gs = h._gpu_state(k)[0]
             for key in ("M", "v", "R", "C"):
                 if getattr(st, key) is not None:
                     getattr(st, key)[:] = gs[key]
@@ -85,7 +85,7 @@ def test_nonfinite_gradients_follow_the_oracle():
         h.opt.sync_status()
         for k in range(len(specs)):
             w0, g, m_prev = pre[k]
-            st = h.ostate[k]
+            st = h.ostate[k][0]
             o = O.tensor_step(w0, g, st, k, h.ohp, t, h.lr, 99)
             where = f"{specs[k].name} step {t}"
             gw = parity.bits16(h.W[k])
@@ -95,7 +95,7 @@ def test_nonfinite_gradients_follow_the_oracle():
             assert diff.size <= 1e-4 * gw.size + 1, f"{where}: {diff.size} weights differ"
             step = np.abs(gw[diff].astype(np.int32) - w0[diff].astype(np.int32))
             assert (step <= 1).all(), f"{where}: weights more than one ulp apart"
-            gs = h._gpu_state(k)
+            gs = h._gpu_state(k)[0]
             for key in ("M", "v", "R", "C"):
                 if getattr(st, key) is not None:
                     scale = None

@@ -225,3 +225,45 @@ def test_row_path_clamp_falls_back_to_phase_b():
     for t in range(1, 4):
         h.step(t, seed=77)
     h.close()
+
+
+def _stacked_workload():
+    """Stacked (E, n, m) tensors on every path: the row path (m = 1024, 4096), the strip
+    path with m % 8 != 0 (each matrix's dither index starts inside a Philox block),
+    an elementwise router stack with an odd matrix size, a momentum stack and a stack
+    of one, with a plain matrix between them so descriptor ids and matrices differ."""
+    B, E, R = WL.TIER_BACKBONE, WL.TIER_EXPERT, WL.TIER_ROUTER
+    specs = [WL.Spec("e4x300x1024", (4, 300, 1024), E), WL.Spec("b100x48", (100, 48), B),
+             WL.Spec("e3x37x100", (3, 37, 100), E), WL.Spec("r3x33x65", (3, 33, 65), R),
+             WL.Spec("b2x64x256", (2, 64, 256), B), WL.Spec("e2x700x4096", (2, 700, 4096), E),
+             WL.Spec("e1x128x512", (1, 128, 512), E), WL.Spec("v999", (999,), B)]
+    return WL.Workload("stacked", specs, WL.HP(), "normal", steps=3)
+
+
+def test_stacked_tensors():
+    """Every matrix of a stack keeps its own factors and clip factor; a matrix whose
+    gradient is zero (mean(R) = 0 at step 1) sits beside live ones."""
+    h = _harness(_stacked_workload())
+    assert h.opt.info(0).stack == 4 and h.opt.info(0).rowpath == 1 and h.opt.info(2).rowpath == 0
+    assert h.opt.info(1).stack == 0
+    for t in range(1, 4):
+        h.load_grads(t)
+        if t == 1:
+            h.G[0][2].zero_()
+            h.G[2][1].zero_()
+        rep = h.step(t, seed=5 + t, grads_loaded=True)
+        assert rep.tensors == sum(s.shape[0] if len(s.shape) == 3 else 1 for s in h.wl.specs)
+    h.close()
+
+
+def test_stacked_appb_experts_full_size_subset():
+    """App. B with the 128 experts of each weight kept as one (128, 4096, 4096) array,
+    in the benchmark's launch configuration; the router and matrices 0, 1, 77 and 127
+    of the first stack are checked."""
+    wl = WL.stack_experts(WL.appb())
+    names = {"b1.router", "experts.w0"}
+    check = [k for k, s in enumerate(wl.specs) if s.name in names]
+    assert len(check) == 2
+    h = _harness(wl, check=check, matrices={check[1]: (0, 1, 77, 127)})
+    h.step(1, seed=3)
+    h.close()

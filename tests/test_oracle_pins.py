@@ -209,6 +209,29 @@ def test_dither_golden():
         assert [int(v, 16) for v in vals] == [int(x) for x in got]
 
 
+def test_dither_index_of_a_stacked_matrix():
+    """Matrix e of a stacked (E, n, m) tensor draws the dithers of its flat position
+    e*n*m + k in the stack (Sec. 3 dithered write-back, the index running over the
+    whole array). An elementwise tier with no clip makes the two halves of a (2n, m)
+    tensor independent, so stepping them as two stacked matrices must reproduce the
+    whole tensor's step bit for bit; n*m = 222 starts the second half inside a block."""
+    rng = np.random.default_rng(21)
+    n, m = 6, 37
+    g = _bf16(rng.normal(0, 1e-3, (2 * n, m)).astype(np.float32)).reshape(-1)
+    w = _bf16(rng.normal(0, 0.02, (2 * n, m)).astype(np.float32)).reshape(-1)
+    hp, lr = _hp(d=1e30), float(F32(1e-3))
+    whole = w.copy()
+    O.tensor_step(whole, g, O.TensorState((2 * n, m), O.TIER_ROUTER), 3, hp, 1, lr, 5)
+    for idx0, want_equal in ((lambda e: e * n * m, True), (lambda e: 0, False)):
+        halves = []
+        for e in range(2):
+            we = w[e * n * m:(e + 1) * n * m].copy()
+            O.tensor_step(we, g[e * n * m:(e + 1) * n * m].copy(), O.TensorState((n, m), O.TIER_ROUTER), 3, hp, 1,
+                          lr, 5, idx0=idx0(e))
+            halves.append(we)
+        assert np.array_equal(np.concatenate(halves), whole) == want_equal
+
+
 def test_dither_uniform_chi2():
     """The 16-bit draws are uniform: chi-square over 256 bins of the top byte and the low byte."""
     r = O.dither16(42, 7, 3, 0, 1 << 20).astype(np.int64)
