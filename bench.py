@@ -125,6 +125,7 @@ def byte_model(opt, n_tensors):
     rc = rc_row = 0
     for k in range(n_tensors):
         i = opt.info(k)
+        E = max(1, i.stack)  # a stack of E matrices: rows / cols are one matrix's
         N += i.numel
         if i.momentum:
             N_mom += i.numel
@@ -134,10 +135,10 @@ def byte_model(opt, n_tensors):
             N_full += i.numel
         elif i.rowpath:
             N_row += i.numel
-            rc_row += i.rows + i.cols
+            rc_row += E * (i.rows + i.cols)
         else:
             N_fact += i.numel
-            rc += i.rows + i.cols
+            rc += E * (i.rows + i.cols)
     step_min = 6 * N + 8 * N_mom + 8 * N_full + 8 * (rc + rc_row)
     kernels = {
         "k_sumsq": 2 * N_fact,                                   # read G of strip-path factored matrices
