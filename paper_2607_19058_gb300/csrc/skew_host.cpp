@@ -353,7 +353,7 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.colp = fact ? (float *)(h->ws + p.ws_colp) : nullptr;
         T.bsc = fact ? (float *)(h->ws + p.ws_bsc) : nullptr;
         T.rsum = fact ? (double *)(h->ws + p.ws_rsum) : nullptr;
-        T.pp = row ? (double *)(h->ws + p.ws_pp) : nullptr;
+        T.pp = row ? (float2 *)(h->ws + p.ws_pp) : nullptr;
         T.rmin = row ? (float *)(h->ws + p.ws_rmin) : nullptr;
         T.fsum = row ? (double *)(h->ws + p.ws_fsum) : nullptr;
         T.fmin = row ? (float *)(h->ws + p.ws_fmin) : nullptr;

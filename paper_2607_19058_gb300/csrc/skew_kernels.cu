@@ -785,35 +785,36 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
             float4 *cp4 = reinterpret_cast<float4 *>(T.colp + base + col);
             cp4[0] = make_float4(cs[v][0].x, cs[v][0].y, cs[v][1].x, cs[v][1].y);
             cp4[1] = make_float4(cs[v][2].x, cs[v][2].y, cs[v][3].x, cs[v][3].y);
-            double2 *pp2 = reinterpret_cast<double2 *>(T.pp + base + col);
+            float4 *pp4 = reinterpret_cast<float4 *>(T.pp + base + col);  // (hi, lo) per column
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-                pp2[q] = make_double2(pair_value(ph[v][q].x, pl[v][q].x), pair_value(ph[v][q].y, pl[v][q].y));
+            for (int q = 0; q < 4; ++q) pp4[q] = make_float4(ph[v][q].x, pl[v][q].x, ph[v][q].y, pl[v][q].y);
         }
     } else {
         // the ring is free (every chunk consumed before the last barrier): stage there
         float *mcs = reinterpret_cast<float *>(sm.buf[0]);        // [TPB][8]
-        double *mpp = reinterpret_cast<double *>(sm.buf[1]);      // [TPB][8]
+        float2 *mpp = reinterpret_cast<float2 *>(sm.buf[1]);      // [TPB][8] (hi, lo)
         __syncthreads();
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             mcs[tid * 8 + 2 * q] = cs[0][q].x;
             mcs[tid * 8 + 2 * q + 1] = cs[0][q].y;
-            mpp[tid * 8 + 2 * q] = pair_value(ph[0][q].x, pl[0][q].x);
-            mpp[tid * 8 + 2 * q + 1] = pair_value(ph[0][q].y, pl[0][q].y);
+            mpp[tid * 8 + 2 * q] = make_float2(ph[0][q].x, pl[0][q].x);
+            mpp[tid * 8 + 2 * q + 1] = make_float2(ph[0][q].y, pl[0][q].y);
         }
         __syncthreads();
         for (int e = tid; e < 8 * V; e += TPB) {  // column e = 8 vi + q
             const int vi = e >> 3, q = e & 7;
             float cc = 0.f;
-            double pq = 0.0;
+            Acc2 pq;
 #pragma unroll
             for (int r = 0; r < RPP; ++r) {
                 cc += mcs[(r * V + vi) * 8 + q];
-                pq += mpp[(r * V + vi) * 8 + q];
+                const float2 h = mpp[(r * V + vi) * 8 + q];
+                pq.add(h.x);
+                pq.lo += h.y;
             }
             T.colp[base + e] = cc;
-            T.pp[base + e] = pq;
+            T.pp[base + e] = make_float2(pq.hi, pq.lo);
         }
     }
     if (zero_row) atomicOr(&S.zflag, 1u);
@@ -878,40 +879,62 @@ __device__ void set_clip(const StepArgs &A, const TensorDev &T, TensorScal &S, d
 // chunk's sum of P_j / C_j. The last item of the tensor forms mean(R) and, when
 // no element can reach the clamp (max_i a_i^2 * max_j b_j^2 <= 1/eps over rows and
 // columns that hold gradient), sum(U^2) = coef^2 * mean(R) * sum_j P_j / C_j and
-// the clip factor; otherwise it queues the tensor for phase B.
+// the clip factor; otherwise it queues the tensor for phase B. P_j and the sums
+// of P_j / C_j are compensated fp32 (hi, lo) pairs: fp64 arithmetic runs at a
+// small fraction of the fp32 rate here, and every term is non-negative, so a
+// pair keeps the sum to about fp64 accuracy and each quotient to one fp32 rounding.
 __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm) {
     const TensorDev &T = A.tensors[t];
     TensorScal &S = A.scal[t];
     const float inf = __int_as_float(0x7F800000);
     const int64_t j = int64_t(local) * kFinChunk + threadIdx.x;
-    double contrib = 0.0;
+    Acc2 contrib;
     float cmin = inf;
     if (threadIdx.x < kFinChunk && j < T.m) {
         const float cs = strided_sum(T.colp + j, T.m, T.rtiles);
-        const double P = strided_sum(T.pp + j, T.m, T.rtiles);
+        Acc2 pa;  // sum over the row tiles of their (hi, lo) partials
+        {
+            const float2 *p = T.pp + j;
+            uint32_t r = 0;
+            for (; r + 8 <= T.rtiles; r += 8) {
+                float2 v[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) v[q] = __ldcg(p + int64_t(r + q) * T.m);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    pa.add(v[q].x);
+                    pa.lo += v[q].y;
+                }
+            }
+            for (; r < T.rtiles; ++r) {
+                const float2 v = __ldcg(p + int64_t(r) * T.m);
+                pa.add(v.x);
+                pa.lo += v.y;
+            }
+        }
+        const float P = isfinite(pa.hi) ? pa.hi + pa.lo : pa.hi;
         const float mean = __fdiv_rn(cs, (float)T.n);
         const float Cn = fmaf(A.b2, T.C[j], A.c2 * mean);
         T.C[j] = Cn;
         T.bsc[j] = __frsqrt_rn(Cn);
-        if (P > 0.0) {
+        if (P > 0.f) {
             if (Cn > 0.f && Cn < inf) {
-                contrib = P / (double)Cn;
+                contrib.add(__fdiv_rn(P, Cn));
                 cmin = Cn;
             } else {
                 atomicOr(&S.zflag, 1u);  // gradient in a column whose C_j is 0 or not finite
             }
-        } else if (!(P == 0.0)) {
+        } else if (!(P == 0.f)) {
             atomicOr(&S.zflag, 1u);  // NaN
         }
     }
-    contrib = block_sum_d(contrib, sm.redd);
 #pragma unroll
     for (int o = 16; o; o >>= 1) cmin = fminf(cmin, __shfl_xor_sync(kAll, cmin, o));
-    if ((threadIdx.x & 31) == 0) sm.red2[threadIdx.x >> 5].x = cmin;
-    __syncthreads();
+    if ((threadIdx.x & 31) == 0) sm.colred[threadIdx.x >> 5] = cmin;
+    const float2 cs2 = block_sum2(contrib, sm.red2);  // its barriers also publish colred
     if (threadIdx.x == 0) {
-        for (int w = 0; w < kThreads / 32; ++w) cmin = fminf(cmin, sm.red2[w].x);
-        T.fsum[local] = contrib;
+        for (int w = 0; w < kThreads / 32; ++w) cmin = fminf(cmin, sm.colred[w]);
+        T.fsum[local] = pair_value(cs2.x, cs2.y);
         T.fmin[local] = cmin;
         sm.last = (atom_add_acq_rel(&S.cntF, 1u) == T.nfc - 1);
     }

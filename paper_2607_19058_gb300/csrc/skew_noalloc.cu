@@ -188,7 +188,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     td.colp = fact ? (float *)(base + o_colp) : nullptr;
     td.bsc = fact ? (float *)(base + o_bsc) : nullptr;
     td.rsum = fact ? (double *)(base + o_rsum) : nullptr;
-    td.pp = row ? (double *)(base + o_pp) : nullptr;
+    td.pp = row ? (float2 *)(base + o_pp) : nullptr;
     td.rmin = row ? (float *)(base + o_rmin) : nullptr;
     td.fsum = row ? (double *)(base + o_fsum) : nullptr;
     td.fmin = row ? (float *)(base + o_fmin) : nullptr;

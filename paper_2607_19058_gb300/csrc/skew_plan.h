@@ -80,7 +80,7 @@ struct TensorDev {
     float *colp;        // factored: column partials of g^2 [rowtiles or rtiles][m]
     float *bsc;         // factored: 1/sqrt(C_j) [m]
     double *rsum;       // factored: sums of R per finalize-row item [nfr] / per row tile [rtiles]
-    double *pp;         // row path: column partials of g^2 / R_i [rtiles][m]
+    float2 *pp;         // row path: column partials of g^2 / R_i [rtiles][m], compensated (hi, lo)
     float *rmin;        // row path: smallest positive R_i per row tile [rtiles]
     double *fsum;       // row path: sum of P_j / C_j per finalize item [nfc]
     float *fmin;        // row path: smallest C_j with P_j > 0 per finalize item [nfc]
