@@ -262,7 +262,6 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
             p.ws_bsc = w;  w = align_up(w + 4 * size_t(p.m), 256);
             p.ws_rsum = w; w = align_up(w + 8 * size_t(p.nfr), 256);
         } else if (p.kind == kKindFactored) {
-            p.ws_colp = w; w = align_up(w + 4 * size_t(p.rtiles) * p.m, 256);
             p.ws_pp = w;   w = align_up(w + 8 * size_t(p.rtiles) * p.m, 256);
             p.ws_bsc = w;  w = align_up(w + 4 * size_t(p.m), 256);
             p.ws_rsum = w; w = align_up(w + 8 * size_t(p.rtiles), 256);
@@ -350,7 +349,7 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.C = p.coff >= 0 ? sf + p.coff : nullptr;
         const bool fact = p.kind == kKindFactored, row = fact && p.rowpath;
         T.rowp = fact && !row ? (float *)(h->ws + p.ws_rowp) : nullptr;
-        T.colp = fact ? (float *)(h->ws + p.ws_colp) : nullptr;
+        T.colp = fact && !row ? (float *)(h->ws + p.ws_colp) : nullptr;
         T.bsc = fact ? (float *)(h->ws + p.ws_bsc) : nullptr;
         T.rsum = fact ? (double *)(h->ws + p.ws_rsum) : nullptr;
         T.pp = row ? (float2 *)(h->ws + p.ws_pp) : nullptr;

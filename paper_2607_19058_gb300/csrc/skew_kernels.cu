@@ -224,6 +224,9 @@ __device__ __forceinline__ double pair_value(float hi, float lo) {
     return isfinite(hi) ? (double)hi + (double)lo : (double)hi;
 }
 
+// The same, rounded to fp32.
+__device__ __forceinline__ float pair_f(float hi, float lo) { return isfinite(hi) ? hi + lo : hi; }
+
 // Compensated accumulator: the running sum is hi + lo.
 struct Acc2 {
     float hi = 0.f, lo = 0.f;
@@ -775,19 +778,19 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         }
         return;
     }
-    // per-tile partials: column sums of g^2 and of g^2 / R_i (the RPP threads that share
-    // a column vector are added in row-in-pass order), the tile's sum and smallest positive R
+    // per-tile partials, (sum of g^2, sum of g^2 / R_i) per column (the RPP threads that
+    // share a column vector are added in row-in-pass order; the compensated sum of
+    // g^2 / R_i is rounded to fp32 once), the tile's sum and smallest positive R
     const int64_t base = int64_t(tile) * 8 * V;
     if constexpr (RPP == 1) {
 #pragma unroll
         for (int v = 0; v < NV; ++v) {
             const int64_t col = 8 * int64_t(v * TPB + lay.vi);
-            float4 *cp4 = reinterpret_cast<float4 *>(T.colp + base + col);
-            cp4[0] = make_float4(cs[v][0].x, cs[v][0].y, cs[v][1].x, cs[v][1].y);
-            cp4[1] = make_float4(cs[v][2].x, cs[v][2].y, cs[v][3].x, cs[v][3].y);
-            float4 *pp4 = reinterpret_cast<float4 *>(T.pp + base + col);  // (hi, lo) per column
+            float4 *pp4 = reinterpret_cast<float4 *>(T.pp + base + col);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) pp4[q] = make_float4(ph[v][q].x, pl[v][q].x, ph[v][q].y, pl[v][q].y);
+            for (int q = 0; q < 4; ++q)
+                pp4[q] = make_float4(cs[v][q].x, pair_f(ph[v][q].x, pl[v][q].x), cs[v][q].y,
+                                     pair_f(ph[v][q].y, pl[v][q].y));
         }
     } else {
         // the ring is free (every chunk consumed before the last barrier): stage there
@@ -813,8 +816,7 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
                 pq.add(h.x);
                 pq.lo += h.y;
             }
-            T.colp[base + e] = cc;
-            T.pp[base + e] = make_float2(pq.hi, pq.lo);
+            T.pp[base + e] = make_float2(cc, pair_f(pq.hi, pq.lo));
         }
     }
     if (zero_row) atomicOr(&S.zflag, 1u);
@@ -891,30 +893,31 @@ __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem 
     Acc2 contrib;
     float cmin = inf;
     if (threadIdx.x < kFinChunk && j < T.m) {
-        const float cs = strided_sum(T.colp + j, T.m, T.rtiles);
-        Acc2 pa;  // sum over the row tiles of their (hi, lo) partials
+        const float Cold = __ldcg(T.C + j);
+        float cs = 0.f;  // sum over the row tiles of g^2 (in tile order) and, compensated, of g^2 / R_i
+        Acc2 pa;
         {
             const float2 *p = T.pp + j;
             uint32_t r = 0;
-            for (; r + 8 <= T.rtiles; r += 8) {
-                float2 v[8];
+            for (; r + 16 <= T.rtiles; r += 16) {
+                float2 v[16];
 #pragma unroll
-                for (int q = 0; q < 8; ++q) v[q] = __ldcg(p + int64_t(r + q) * T.m);
+                for (int q = 0; q < 16; ++q) v[q] = __ldcg(p + int64_t(r + q) * T.m);
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    pa.add(v[q].x);
-                    pa.lo += v[q].y;
+                for (int q = 0; q < 16; ++q) {
+                    cs += v[q].x;
+                    pa.add(v[q].y);
                 }
             }
             for (; r < T.rtiles; ++r) {
                 const float2 v = __ldcg(p + int64_t(r) * T.m);
-                pa.add(v.x);
-                pa.lo += v.y;
+                cs += v.x;
+                pa.add(v.y);
             }
         }
-        const float P = isfinite(pa.hi) ? pa.hi + pa.lo : pa.hi;
+        const float P = pair_f(pa.hi, pa.lo);
         const float mean = __fdiv_rn(cs, (float)T.n);
-        const float Cn = fmaf(A.b2, T.C[j], A.c2 * mean);
+        const float Cn = fmaf(A.b2, Cold, A.c2 * mean);
         T.C[j] = Cn;
         T.bsc[j] = __frsqrt_rn(Cn);
         if (P > 0.f) {

@@ -149,7 +149,6 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
         o_bsc = off;  off = align256(off + 4 * size_t(m));
         o_rsum = off; off = align256(off + 8 * size_t(G.nfr));
     } else if (row) {
-        o_colp = off; off = align256(off + 4 * size_t(G.rtiles) * m);
         o_pp = off;   off = align256(off + 8 * size_t(G.rtiles) * m);
         o_bsc = off;  off = align256(off + 4 * size_t(m));
         o_rsum = off; off = align256(off + 8 * size_t(G.rtiles));
@@ -185,7 +184,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     td.R = R;
     td.C = Cc;
     td.rowp = fact && !row ? (float *)(base + o_rowp) : nullptr;
-    td.colp = fact ? (float *)(base + o_colp) : nullptr;
+    td.colp = fact && !row ? (float *)(base + o_colp) : nullptr;
     td.bsc = fact ? (float *)(base + o_bsc) : nullptr;
     td.rsum = fact ? (double *)(base + o_rsum) : nullptr;
     td.pp = row ? (float2 *)(base + o_pp) : nullptr;

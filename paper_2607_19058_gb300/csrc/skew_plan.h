@@ -77,10 +77,10 @@ struct TensorDev {
     float *R;           // row factor (n) or null
     float *C;           // column factor (m) or null
     float *rowp;        // strip path: row partials [strips][n]
-    float *colp;        // factored: column partials of g^2 [rowtiles or rtiles][m]
+    float *colp;        // strip path: column partials of g^2 [rowtiles][m]
     float *bsc;         // factored: 1/sqrt(C_j) [m]
     double *rsum;       // factored: sums of R per finalize-row item [nfr] / per row tile [rtiles]
-    float2 *pp;         // row path: column partials of g^2 / R_i [rtiles][m], compensated (hi, lo)
+    float2 *pp;         // row path: per row tile and column, (sum of g^2, sum of g^2 / R_i) [rtiles][m]
     float *rmin;        // row path: smallest positive R_i per row tile [rtiles]
     double *fsum;       // row path: sum of P_j / C_j per finalize item [nfc]
     float *fmin;        // row path: smallest C_j with P_j > 0 per finalize item [nfc]
