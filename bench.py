@@ -205,8 +205,10 @@ def oracle_sample_specs(wl, target_params):
 
 def time_oracle(wl, tids, inputs, step, lr, seed):
     import oracle as O
+    from paper_2607_19058_gb300 import workloads as WL
     hpd = wl.hp
-    ohp = O.hparams(hpd.beta1, hpd.beta2, hpd.eps, hpd.clip_d, hpd.weight_decay)
+    ohp = O.hparams(hpd.beta1, hpd.beta2, hpd.eps, hpd.clip_d, hpd.weight_decay,
+                    annealed=hpd.policy == WL.POLICY_ADAFACTOR)
     states = {k: O.TensorState(wl.specs[k].shape, wl.specs[k].tier, hpd.policy, wl.specs[k].no_decay) for k in tids}
     t0 = time.perf_counter()
     for k in tids:

@@ -67,6 +67,11 @@ extern "C" {
 #define SKEW_POLICY_EXPERT_MOMENTUM 1 /* "+ momentum on experts"                        */
 #define SKEW_POLICY_FACTORED_ROUTER 2 /* "factored router"                              */
 #define SKEW_POLICY_UNIFORM 3         /* "uniform (momentum + factored)" on every tier  */
+/* The Adafactor comparator (Sec. 5, Table 4 and its footnote, App. A; Shazeer &
+ * Stern 2018): every matrix factored (the router too), vectors exact, no momentum, the
+ * second-moment decay annealed as beta2_t = 1 - t^-0.8 (beta1 and beta2 are then
+ * unused) and no bias correction; the same clipping, decay and write-back. */
+#define SKEW_POLICY_ADAFACTOR 4
 
 /* ---- per-tensor flags ------------------------------------------------------ */
 #define SKEW_F_NO_DECAY 1u /* exempt this tensor from weight decay (the router always is) */

@@ -24,7 +24,7 @@ LIB = os.path.join(HERE, "libskew_oracle.so")
 
 KIND_FULL, KIND_FACTORED = 0, 1
 TIER_BACKBONE, TIER_EXPERT, TIER_ROUTER = 0, 1, 2
-POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM = 0, 1, 2, 3
+POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM, POLICY_ADAFACTOR = 0, 1, 2, 3, 4
 
 _lock = threading.Lock()
 _lib = None
@@ -52,7 +52,7 @@ class _Tensor(C.Structure):
 
 class _HParams(C.Structure):
     _fields_ = [("beta1", C.c_double), ("beta2", C.c_double), ("eps", C.c_double),
-                ("clip_d", C.c_double), ("weight_decay", C.c_double)]
+                ("clip_d", C.c_double), ("weight_decay", C.c_double), ("annealed", C.c_int32)]
 
 
 def lib():
@@ -150,10 +150,11 @@ class TensorState:
         return sum(a.nbytes for a in (self.M, self.v, self.R, self.C) if a is not None)
 
 
-def hparams(beta1, beta2, eps, clip_d, weight_decay):
-    """The fp32 hyper-parameters widened to double (both sides use the fp32 values)."""
+def hparams(beta1, beta2, eps, clip_d, weight_decay, annealed: bool = False):
+    """The fp32 hyper-parameters widened to double (both sides use the fp32 values).
+    `annealed`: the Adafactor comparator's decay 1 - t^-0.8 without bias correction."""
     f = lambda x: float(np.float32(x))
-    return _HParams(f(beta1), f(beta2), f(eps), f(clip_d), f(weight_decay))
+    return _HParams(f(beta1), f(beta2), f(eps), f(clip_d), f(weight_decay), int(annealed))
 
 
 def tensor_step(w_bits: np.ndarray, g_bits: np.ndarray, st: TensorState, tid: int, hp, step: int,

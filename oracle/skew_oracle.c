@@ -132,7 +132,8 @@ uint16_t so_sr_bf16(float x, uint16_t r)
 /* Tier policy (Sec. 3 "The tiers", Algorithm 1, Table 3 variants).          */
 /* ------------------------------------------------------------------------ */
 enum { SO_TIER_BACKBONE = 0, SO_TIER_EXPERT = 1, SO_TIER_ROUTER = 2 };
-enum { SO_POLICY_TIERED = 0, SO_POLICY_EXPERT_MOMENTUM = 1, SO_POLICY_FACTORED_ROUTER = 2, SO_POLICY_UNIFORM = 3 };
+enum { SO_POLICY_TIERED = 0, SO_POLICY_EXPERT_MOMENTUM = 1, SO_POLICY_FACTORED_ROUTER = 2, SO_POLICY_UNIFORM = 3,
+       SO_POLICY_ADAFACTOR = 4 };
 enum { SO_KIND_FULL = 0, SO_KIND_FACTORED = 1 };
 
 /*
@@ -143,6 +144,8 @@ enum { SO_KIND_FULL = 0, SO_KIND_FACTORED = 1 };
  * momentum: backbone tensors carry fp32 momentum; experts only under the
  *           "+ momentum on experts" and "uniform" variants; the router only
  *           under "uniform".
+ * The Adafactor comparator (Sec. 5 and its footnote, App. A "no momentum")
+ * factors every matrix, the router too, and keeps no momentum anywhere.
  * decay:    every tier but the router ("no weight decay" for the router),
  *           unless the caller exempts the tensor.
  * Returns 0, or -1 for an unknown tier / policy / ndim.
@@ -150,16 +153,19 @@ enum { SO_KIND_FULL = 0, SO_KIND_FACTORED = 1 };
 int so_resolve(int ndim, int tier, int policy, int no_decay, int *kind, int *momentum, int *decay)
 {
     if (ndim != 1 && ndim != 2) return -1;
-    if (tier < 0 || tier > 2 || policy < 0 || policy > 3) return -1;
+    if (tier < 0 || tier > 2 || policy < 0 || policy > 4) return -1;
     int k;
     if (ndim == 1)
         k = SO_KIND_FULL;
-    else if (tier == SO_TIER_ROUTER && policy != SO_POLICY_FACTORED_ROUTER && policy != SO_POLICY_UNIFORM)
+    else if (tier == SO_TIER_ROUTER && policy != SO_POLICY_FACTORED_ROUTER && policy != SO_POLICY_UNIFORM &&
+             policy != SO_POLICY_ADAFACTOR)
         k = SO_KIND_FULL;
     else
         k = SO_KIND_FACTORED;
     int mo;
-    if (tier == SO_TIER_BACKBONE)
+    if (policy == SO_POLICY_ADAFACTOR)
+        mo = 0;
+    else if (tier == SO_TIER_BACKBONE)
         mo = 1;
     else if (tier == SO_TIER_EXPERT)
         mo = (policy == SO_POLICY_EXPERT_MOMENTUM || policy == SO_POLICY_UNIFORM);
@@ -231,6 +237,8 @@ typedef struct {
 
 typedef struct {
     double beta1, beta2, eps, clip_d, weight_decay;
+    int32_t annealed;   /* 1: the Adafactor comparator's decay beta2_t = 1 - t^-0.8 */
+                        /* (as an fp32 value) and no bias correction; beta2 unused  */
 } so_hparams_t;
 
 /*
@@ -245,9 +253,15 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
 {
     if (!T || !hp || t < 1 || T->n < 1 || T->m < 1) return -1;
     const int64_t n = T->n, m = T->m, numel = n * m;
-    const double b1 = hp->beta1, b2 = hp->beta2;
-    const double bc1 = 1.0 - so_powi(b1, t);           /* 1 - beta1^t        */
-    const double s2 = sqrt(1.0 - so_powi(b2, t));      /* sqrt(1 - beta2^t)  */
+    const double b1 = hp->beta1;
+    double b2 = hp->beta2;
+    double bc1 = 1.0 - so_powi(b1, t);           /* 1 - beta1^t        */
+    double s2 = sqrt(1.0 - so_powi(b2, t));      /* sqrt(1 - beta2^t)  */
+    if (hp->annealed) {                          /* Adafactor: beta2_t = 1 - t^-0.8, no correction */
+        b2 = (double)(float)(1.0 - pow((double)t, -0.8));
+        bc1 = 1.0;
+        s2 = 1.0;
+    }
 
     double *U = (double *)malloc((size_t)numel * sizeof(double));
     if (!U) return -1;

@@ -89,21 +89,13 @@ static int cuda_fail(skew_handle_t *h, cudaError_t e, const char *what) {
     return fail(h, SKEW_ECUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-// Tier policy: (kind, momentum, decay) of one tensor.
+// Tier policy: (kind, momentum, decay) of one tensor (resolve_policy).
 static void resolve(int ndim, int tier, int policy, uint32_t flags, TPlan &p) {
-    if (ndim == 1)
-        p.kind = kKindFull;  // Algorithm 1: a vector keeps the full second moment
-    else if (tier == SKEW_TIER_ROUTER && policy != SKEW_POLICY_FACTORED_ROUTER && policy != SKEW_POLICY_UNIFORM)
-        p.kind = kKindFull;  // the router keeps the exact second moment
-    else
-        p.kind = kKindFactored;  // Eq. 1
-    if (tier == SKEW_TIER_BACKBONE)
-        p.momentum = 1;
-    else if (tier == SKEW_TIER_EXPERT)
-        p.momentum = (policy == SKEW_POLICY_EXPERT_MOMENTUM || policy == SKEW_POLICY_UNIFORM);
-    else
-        p.momentum = (policy == SKEW_POLICY_UNIFORM);
-    p.decay = (tier != SKEW_TIER_ROUTER) && !(flags & SKEW_F_NO_DECAY);
+    uint32_t kind, momentum, decay;
+    resolve_policy(ndim, tier, policy, flags, kind, momentum, decay);
+    p.kind = (int)kind;
+    p.momentum = (int)momentum;
+    p.decay = (int)decay;
 }
 
 // Tile geometry (plan_geometry): strip tiles of (tile_rows rows) x (8*LC
@@ -138,7 +130,7 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
     if (!finite(H.eps) || !(H.eps > 0.f)) return fail(nullptr, SKEW_EINVAL, "eps must be finite and > 0");
     if (!finite(H.clip_d) || !(H.clip_d > 0.f)) return fail(nullptr, SKEW_EINVAL, "clip_d must be finite and > 0");
     if (!finite(H.weight_decay) || H.weight_decay < 0.f) return fail(nullptr, SKEW_EINVAL, "weight_decay must be finite and >= 0");
-    if (H.policy < SKEW_POLICY_TIERED || H.policy > SKEW_POLICY_UNIFORM) return fail(nullptr, SKEW_EINVAL, "unknown policy %d", H.policy);
+    if (H.policy < SKEW_POLICY_TIERED || H.policy > SKEW_POLICY_ADAFACTOR) return fail(nullptr, SKEW_EINVAL, "unknown policy %d", H.policy);
 
     skew_handle *h = new (std::nothrow) skew_handle();
     if (!h) return fail(nullptr, SKEW_ENOMEM, "out of host memory");
@@ -430,9 +422,7 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
     if (h->t.empty()) return SKEW_OK;
     cudaStream_t s = (cudaStream_t)stream;
     const skew_hparams_t &H = h->hp;
-    const double t = (double)step;
-    const double bc1 = 1.0 - std::pow((double)H.beta1, t);
-    const double s2 = std::sqrt(1.0 - std::pow((double)H.beta2, t));
+    const StepCoefs k = step_coefs(H, step);
 
     StepArgs a{};
     a.tensors = reinterpret_cast<const TensorDev *>(h->ws + h->ws_tens);
@@ -440,15 +430,15 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
     a.err = reinterpret_cast<uint32_t *>(h->ws + h->ws_err);
     a.fb = reinterpret_cast<uint32_t *>(h->ws + h->ws_fb);
     a.b1 = H.beta1;
-    a.b2 = H.beta2;
+    a.b2 = k.b2;
     a.c1 = (float)(1.0 - (double)H.beta1);
-    a.c2 = (float)(1.0 - (double)H.beta2);
+    a.c2 = k.c2;
     a.ce = (float)(1.0 / std::sqrt((double)H.eps));
     a.wdf = (float)(1.0 - (double)lr * (double)H.weight_decay);
     a.lr = lr;
     a.clip_d = H.clip_d;
-    a.coef_mom = s2 / bc1;
-    a.coef_plain = s2;
+    a.coef_mom = k.coef_mom;
+    a.coef_plain = k.coef_plain;
     a.step_lo = (uint32_t)(uint64_t)step;
     a.seed_lo = (uint32_t)seed;
     a.seed_hi = (uint32_t)(seed >> 32);

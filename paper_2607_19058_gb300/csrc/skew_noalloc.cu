@@ -88,7 +88,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     if (!std::isfinite(H.eps) || !(H.eps > 0.f)) return SKEW_EINVAL;
     if (!std::isfinite(H.clip_d) || !(H.clip_d > 0.f)) return SKEW_EINVAL;
     if (!std::isfinite(H.weight_decay) || H.weight_decay < 0.f) return SKEW_EINVAL;
-    if (H.policy < SKEW_POLICY_TIERED || H.policy > SKEW_POLICY_UNIFORM) return SKEW_EINVAL;
+    if (H.policy < SKEW_POLICY_TIERED || H.policy > SKEW_POLICY_ADAFACTOR) return SKEW_EINVAL;
     if (step < 1) return SKEW_EINVAL;
     if (!std::isfinite(lr) || lr < 0.f) return SKEW_EINVAL;
     const int64_t n = rows, m = ndim == 2 ? cols : 1;
@@ -98,17 +98,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
 
     // ---- tier policy (as the planner's, Sec. 3 "The tiers" / Table 3) -------------
     uint32_t kind, momentum, decay;
-    if (ndim == 1 || (tier == SKEW_TIER_ROUTER && H.policy != SKEW_POLICY_FACTORED_ROUTER && H.policy != SKEW_POLICY_UNIFORM))
-        kind = kKindFull;
-    else
-        kind = kKindFactored;
-    if (tier == SKEW_TIER_BACKBONE)
-        momentum = 1;
-    else if (tier == SKEW_TIER_EXPERT)
-        momentum = (H.policy == SKEW_POLICY_EXPERT_MOMENTUM || H.policy == SKEW_POLICY_UNIFORM);
-    else
-        momentum = (H.policy == SKEW_POLICY_UNIFORM);
-    decay = (tier != SKEW_TIER_ROUTER) && !(flags & SKEW_F_NO_DECAY);
+    resolve_policy(ndim, tier, H.policy, flags, kind, momentum, decay);
 
     // ---- caller's state: [M][v][R][C] of this tensor, exactly the closed form -----
     const int64_t state_floats = (momentum ? numel : 0) + (kind == kKindFull ? numel : n + m);
@@ -216,24 +206,22 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     td.rtiles = G.rtiles;
 
     // ---- per-step scalars, as skew_step forms them ------------------------------------
-    const double t = (double)step;
-    const double bc1 = 1.0 - std::pow((double)H.beta1, t);
-    const double s2 = std::sqrt(1.0 - std::pow((double)H.beta2, t));
+    const StepCoefs k = step_coefs(H, step);
     StepArgs a{};
     a.tensors = (const TensorDev *)(base + o_tens);
     a.scal = (TensorScal *)(base + o_scal);
     a.err = (uint32_t *)(base + o_err);
     a.fb = (uint32_t *)(base + o_fb);
     a.b1 = H.beta1;
-    a.b2 = H.beta2;
+    a.b2 = k.b2;
     a.c1 = (float)(1.0 - (double)H.beta1);
-    a.c2 = (float)(1.0 - (double)H.beta2);
+    a.c2 = k.c2;
     a.ce = (float)(1.0 / std::sqrt((double)H.eps));
     a.wdf = (float)(1.0 - (double)lr * (double)H.weight_decay);
     a.lr = lr;
     a.clip_d = H.clip_d;
-    a.coef_mom = s2 / bc1;
-    a.coef_plain = s2;
+    a.coef_mom = k.coef_mom;
+    a.coef_plain = k.coef_plain;
     a.step_lo = (uint32_t)(uint64_t)step;
     a.seed_lo = (uint32_t)seed;
     a.seed_hi = (uint32_t)(seed >> 32);

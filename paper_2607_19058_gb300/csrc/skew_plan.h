@@ -3,8 +3,11 @@
 // libskewadam. Not part of the public ABI.
 #pragma once
 
+#include <math.h>
 #include <stdint.h>
 #include <vector_types.h>
+
+#include "skewadam.h"
 
 namespace skew {
 
@@ -25,6 +28,54 @@ constexpr int kRowChunks = 32;
 constexpr int kRowStages = 3;
 
 enum Kind : uint32_t { kKindFull = 0, kKindFactored = 1 };
+
+// Tier policy of one tensor (Sec. 3 "The tiers", Algorithm 1, the Table 3
+// variants, and the Adafactor comparator of Sec. 5 / App. A): a vector keeps the exact
+// second moment; the router too unless the variant factors it; every other matrix
+// is factored (Eq. 1). Momentum: the backbone; experts under "+ momentum on
+// experts" and "uniform"; the router under "uniform"; nothing under Adafactor.
+// Weight decay: every tier but the router, unless the caller exempts the tensor.
+inline void resolve_policy(int ndim, int tier, int policy, uint32_t flags, uint32_t &kind, uint32_t &momentum,
+                           uint32_t &decay) {
+    const bool router_factored = policy == SKEW_POLICY_FACTORED_ROUTER || policy == SKEW_POLICY_UNIFORM ||
+                                 policy == SKEW_POLICY_ADAFACTOR;
+    kind = (ndim == 1 || (tier == SKEW_TIER_ROUTER && !router_factored)) ? kKindFull : kKindFactored;
+    if (policy == SKEW_POLICY_ADAFACTOR)
+        momentum = 0;
+    else if (tier == SKEW_TIER_BACKBONE)
+        momentum = 1;
+    else if (tier == SKEW_TIER_EXPERT)
+        momentum = (policy == SKEW_POLICY_EXPERT_MOMENTUM || policy == SKEW_POLICY_UNIFORM);
+    else
+        momentum = (policy == SKEW_POLICY_UNIFORM);
+    decay = (tier != SKEW_TIER_ROUTER) && !(flags & SKEW_F_NO_DECAY);
+}
+
+// Second-moment decay (fp32, with 1 - beta2 formed from it in fp64) and the update
+// coefficients of step t: sqrt(1 - beta2^t) / (1 - beta1^t) with momentum and
+// sqrt(1 - beta2^t) without (Algorithm 1's bias corrections). The Adafactor
+// comparator anneals the decay, beta2_t = 1 - t^-0.8, and has no bias correction.
+struct StepCoefs {
+    float b2, c2;
+    double coef_mom, coef_plain;
+};
+
+inline StepCoefs step_coefs(const skew_hparams_t &H, int64_t step) {
+    const double t = (double)step;
+    StepCoefs c;
+    if (H.policy == SKEW_POLICY_ADAFACTOR) {
+        c.b2 = (float)(1.0 - pow(t, -0.8));
+        c.c2 = (float)(1.0 - (double)c.b2);
+        c.coef_mom = c.coef_plain = 1.0;
+    } else {
+        const double s2 = sqrt(1.0 - pow((double)H.beta2, t));
+        c.b2 = H.beta2;
+        c.c2 = (float)(1.0 - (double)H.beta2);
+        c.coef_mom = s2 / (1.0 - pow((double)H.beta1, t));
+        c.coef_plain = s2;
+    }
+    return c;
+}
 
 // Tile geometry of one tensor (shared by every entry point, so that the same
 // tensor is always cut the same way and results are bit-identical).

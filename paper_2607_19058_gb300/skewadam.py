@@ -21,7 +21,7 @@ LIB_PATH = os.path.join(HERE, "libskewadam.so")
 SKEW_OK, SKEW_EINVAL, SKEW_ENOMEM, SKEW_ECUDA, SKEW_ETIMEOUT, SKEW_ESTATE, SKEW_ETOOBIG = 0, -1, -2, -3, -4, -5, -6
 NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 TIER_BACKBONE, TIER_EXPERT, TIER_ROUTER = 0, 1, 2
-POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM = 0, 1, 2, 3
+POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM, POLICY_ADAFACTOR = 0, 1, 2, 3, 4
 F_NO_DECAY = 1
 KIND_FULL, KIND_FACTORED = 0, 1
 

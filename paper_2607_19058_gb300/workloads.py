@@ -31,7 +31,7 @@ from typing import List, Optional, Sequence, Tuple
 import torch
 
 TIER_BACKBONE, TIER_EXPERT, TIER_ROUTER = 0, 1, 2
-POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM = 0, 1, 2, 3
+POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM, POLICY_ADAFACTOR = 0, 1, 2, 3, 4
 
 
 @dataclasses.dataclass(frozen=True)
@@ -154,6 +154,12 @@ def ablation() -> Workload:
     return Workload("ablation", specs, HP(policy=POLICY_EXPERT_MOMENTUM), "normal", steps=20, n_experts=128)
 
 
+def adafactor() -> Workload:
+    """The App. B shapes under the Adafactor comparator (Sec. 5, App. A): every matrix
+    factored, no momentum, beta2_t = 1 - t^-0.8."""
+    return Workload("adafactor", _appb_specs(), HP(policy=POLICY_ADAFACTOR), "normal", steps=20, n_experts=128)
+
+
 def small() -> Workload:
     """A 573M-parameter cut of the App. B set (32 experts, a 4096^2 and a 1024x4096 backbone
     matrix, 2 norm vectors, the router): 2.3 GB of weights + gradients, well above L2,
@@ -182,7 +188,7 @@ def stack_experts(wl: Workload) -> Workload:
 
 
 WORKLOADS = {"small": small, "toy": toy, "slice": slice_, "appb": appb, "literal": literal, "skewed": skewed,
-             "ablation": ablation}
+             "ablation": ablation, "adafactor": adafactor}
 
 
 def get(name: str) -> Workload:

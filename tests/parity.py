@@ -175,7 +175,8 @@ class Harness:
         self.check = list(range(len(wl.specs))) if check is None else list(check)
         self.ostate = {k: {e: O.TensorState(self._mat_shape(k), wl.specs[k].tier, hpd["policy"], wl.specs[k].no_decay)
                            for e in (matrices or {}).get(k, range(self._stack(k)))} for k in self.check}
-        self.ohp = O.hparams(hpd["beta1"], hpd["beta2"], hpd["eps"], hpd["clip_d"], hpd["weight_decay"])
+        self.ohp = O.hparams(hpd["beta1"], hpd["beta2"], hpd["eps"], hpd["clip_d"], hpd["weight_decay"],
+                             annealed=hpd["policy"] == WL.POLICY_ADAFACTOR)
         self.lr = hpd["lr"]
 
     def load_grads(self, t: int):

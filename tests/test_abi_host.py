@@ -80,7 +80,7 @@ def _descs(wl, base=0x100000):
 @pytest.mark.parametrize("name", ["toy", "slice", "appb", "literal", "skewed", "ablation"])
 def test_state_bytes_is_closed_form(name):
     wl = WL.get(name)
-    for policy in (wl.hp.policy, S.POLICY_UNIFORM, S.POLICY_FACTORED_ROUTER):
+    for policy in (wl.hp.policy, S.POLICY_UNIFORM, S.POLICY_FACTORED_ROUTER, S.POLICY_ADAFACTOR):
         h = S.skew_create(_descs(wl), S.hparams(policy=policy))
         want = O.state_bytes([(s.shape, s.tier) for s in wl.specs], policy)
         assert S.skew_state_bytes(h) == want
@@ -183,7 +183,7 @@ def test_create_rejects_bad_extents(shape):
 
 
 @pytest.mark.parametrize("hp", [dict(beta1=1.0), dict(beta2=-0.1), dict(eps=0.0), dict(eps=float("nan")),
-                                dict(clip_d=0.0), dict(weight_decay=-1.0), dict(policy=7), dict(beta1=float("inf"))])
+                                dict(clip_d=0.0), dict(weight_decay=-1.0), dict(policy=5), dict(beta1=float("inf"))])
 def test_create_rejects_bad_hparams(hp):
     with pytest.raises(S.SkewError) as e:
         S.skew_create([_one()], S.hparams(**hp))

@@ -267,3 +267,18 @@ def test_stacked_appb_experts_full_size_subset():
     h = _harness(wl, check=check, matrices={check[1]: (0, 1, 77, 127)})
     h.step(1, seed=3)
     h.close()
+
+
+def test_adafactor_comparator():
+    """The Adafactor comparator (every matrix factored, no momentum, beta2_t = 1 - t^-0.8, no
+    bias correction) on the toy set (strip path, exact vectors, zero-gradient experts at t = 1)
+    and on the whole-row path, over steps whose decay changes every step."""
+    h = _harness(WL.toy(), hp_override=dict(policy=WL.POLICY_ADAFACTOR))
+    assert all(h.opt.info(k).momentum == 0 for k in range(len(h.wl.specs)))
+    for t in range(1, 5):
+        h.step(t, seed=t)
+    h.close()
+    h = _harness(_row_path_workload(), hp_override=dict(policy=WL.POLICY_ADAFACTOR))
+    for t in range(1, 4):
+        h.step(t, seed=11 * t)
+    h.close()

@@ -98,6 +98,53 @@ def test_state_bytes_table3_variants():
     assert round(un / 2**30, 2) == 25.29
 
 
+def test_state_bytes_adafactor():
+    """Sec. 5 / Table 4: uniform Adafactor carries about 12 MB (0.01 GB): R and C of every
+    matrix (the router's too) and the vectors' full v, no momentum. Hand sum over the App. B
+    shapes: 384 experts, embedding, positions, 2 x attention, dense FFN, router, 10 vectors."""
+    ad = O.state_bytes(_specs(WL.appb()), O.POLICY_ADAFACTOR)
+    want = 4 * (384 * (4096 + 4096) + (50304 + 4096) + (256 + 4096) + 2 * (2 * 8192 + 2 * 5120)
+                + 3 * 8192 + (4096 + 128) + 10 * 4096)
+    assert ad == want == 13_309_952
+    assert round(ad / 1e9, 2) == 0.01 and 12 <= ad / 2**20 < 13
+
+
+def test_adafactor_annealed_decay_closed_forms():
+    """Adafactor comparator (Sec. 5 footnote: decay 1 - t^-0.8; App. A: no momentum; no bias
+    correction). beta2_1 = 0, so at t = 1 a vector's v is g^2 and U = sign(g). A zero gradient
+    at t = 1 and g at t = 2 give v = (1 - beta2_2) g^2 with 1 - beta2_2 ~ 2^-0.8: U = g / sqrt(v),
+    RMS = 1/sqrt(1 - beta2_2) ~ 2^0.4 > 1, and the clip turns the update into sign(g)."""
+    rng = np.random.default_rng(12)
+    n = 512
+    g = _bf16(rng.normal(0, 1e-3, n).astype(np.float32))
+    g[g == 0] = _bf16(np.float32(1e-3))
+    w = _bf16(rng.normal(0, 0.02, n).astype(np.float32))
+    lr = float(F32(1e-3))
+    hp = O.hparams(0.9, 0.999, 1e-30, 1.0, 0.0, annealed=True)
+    gd = _f(g).astype(np.float64)
+    st = O.TensorState((n,), O.TIER_BACKBONE, O.POLICY_ADAFACTOR)
+    assert st.momentum == 0 and st.kind == O.KIND_FULL
+    w1 = w.copy()
+    o = O.tensor_step(w1, g, st, 0, hp, 1, lr, 3, want_x=True)
+    assert np.array_equal(st.v, (gd * gd).astype(np.float32))
+    assert abs(o["rms"] - 1.0) < 1e-7 and o["kappa"] == 1.0
+    want = (_f(w).astype(np.float64) - lr * np.sign(gd)).astype(np.float32)
+    assert np.max(np.abs(o["x"].astype(np.float64) - want)) <= 4e-7 * lr + np.spacing(want).max()
+    # t = 1 with a zero gradient, t = 2 with g
+    st = O.TensorState((n,), O.TIER_BACKBONE, O.POLICY_ADAFACTOR)
+    w2 = w.copy()
+    O.tensor_step(w2, np.zeros_like(g), st, 0, hp, 1, lr, 3)
+    w2_pre = w2.copy()
+    o = O.tensor_step(w2, g, st, 0, hp, 2, lr, 3, want_x=True)
+    c2 = 1.0 - float(np.float32(1.0 - 2.0 ** -0.8))
+    assert abs(c2 - 2.0 ** -0.8) < 1e-7
+    assert np.array_equal(st.v, (c2 * gd * gd).astype(np.float32))
+    assert abs(o["rms"] - 1.0 / np.sqrt(c2)) < 2e-7 * o["rms"]
+    assert abs(o["kappa"] - np.sqrt(c2)) < 2e-7
+    want = (_f(w2_pre).astype(np.float64) - lr * np.sign(gd)).astype(np.float32)
+    assert np.max(np.abs(o["x"].astype(np.float64) - want)) <= 4e-7 * lr + np.spacing(want).max()
+
+
 def test_state_bytes_other_shape_sets():
     """Hand-summed closed form for the toy, slice, literal and ablation sets."""
     assert O.state_bytes(_specs(WL.toy())) == 356_096
@@ -118,8 +165,16 @@ def test_tier_policy():
     assert O.resolve(2, O.TIER_ROUTER, O.POLICY_FACTORED_ROUTER) == (FACT, 0, 0)
     assert O.resolve(2, O.TIER_ROUTER, O.POLICY_UNIFORM) == (FACT, 1, 0)
     assert O.resolve(2, O.TIER_EXPERT, no_decay=True) == (FACT, 0, 0)
+    # the Adafactor comparator (Sec. 5, App. A): every matrix factored, no momentum anywhere
+    AD = O.POLICY_ADAFACTOR
+    assert O.resolve(2, O.TIER_BACKBONE, AD) == (FACT, 0, 1)
+    assert O.resolve(1, O.TIER_BACKBONE, AD) == (FULL, 0, 1)
+    assert O.resolve(2, O.TIER_EXPERT, AD) == (FACT, 0, 1)
+    assert O.resolve(2, O.TIER_ROUTER, AD) == (FACT, 0, 0)
     with pytest.raises(ValueError):
         O.resolve(3, O.TIER_EXPERT)
+    with pytest.raises(ValueError):
+        O.resolve(2, O.TIER_EXPERT, 5)
 
 
 # --------------------------------------------------------------------------
