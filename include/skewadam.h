@@ -75,6 +75,10 @@ extern "C" {
 
 /* ---- per-tensor flags ------------------------------------------------------ */
 #define SKEW_F_NO_DECAY 1u /* exempt this tensor from weight decay (the router always is) */
+/* Weights and gradient are fp32 (4-byte aligned), as the paper keeps the norms and
+ * the router (App. A): the new weight is the fp32 update itself, with no dithered
+ * cast. Such a tensor takes the scalar tile path (it is small). */
+#define SKEW_F_FP32 2u
 
 /* ---- second-moment kinds reported by skew_tensor_info ----------------------- */
 #define SKEW_KIND_FULL 0     /* exact second moment v (router, vectors)  */
@@ -85,12 +89,13 @@ typedef struct skew_handle skew_handle_t; /* opaque */
 /*
  * One parameter tensor. The tensor id used by the dither is its index in the
  * array passed to skew_create.
- *   weight : device pointer to the bf16 weights, contiguous row-major, updated
- *            in place by skew_step; 2-byte aligned (16-byte alignment enables
- *            the vectorised path). Borrowed: must stay valid while the handle
+ *   weight : device pointer to the bf16 weights (fp32 with SKEW_F_FP32),
+ *            contiguous row-major, updated in place by skew_step; 2-byte
+ *            aligned, 4-byte for fp32 (16-byte alignment enables the
+ *            vectorised bf16 path). Borrowed: must stay valid while the handle
  *            is bound.
- *   grad   : device pointer to the bf16 gradient, same shape and layout; read
- *            only. Borrowed like `weight`.
+ *   grad   : device pointer to the gradient, the weights' type, shape and
+ *            layout; read only. Borrowed like `weight`.
  *   shape  : shape[0] = rows n (>= 1); shape[1] = columns m (>= 1) when
  *            ndim >= 2, ignored when ndim == 1.
  *   ndim   : 1 (vector), 2 (matrix) or 3 (a stack of `stack` matrices of
@@ -260,7 +265,8 @@ const char *skew_kernel_name(int32_t k);
  * whole-row partials take more room); larger tensors are rejected with
  * SKEW_ETOOBIG before any work is enqueued.
  *
- * Arguments: weight / grad as in skew_param_desc_t (device, bf16, row-major);
+ * Arguments: weight / grad as in skew_param_desc_t (device, bf16 or with
+ * SKEW_F_FP32 fp32, row-major);
  * ndim, rows, cols, tier, flags as in skew_param_desc_t; hp as for
  * skew_create; state: this tensor's fp32 state, exactly state_bytes =
  * 4 * ((momentum ? numel : 0) + (full second moment ? numel : rows + cols))

@@ -46,7 +46,7 @@ class _Tensor(C.Structure):
         ("w", C.c_void_p), ("g", C.c_void_p), ("M", C.c_void_p), ("v", C.c_void_p),
         ("R", C.c_void_p), ("C", C.c_void_p), ("n", C.c_int64), ("m", C.c_int64),
         ("kind", C.c_int32), ("momentum", C.c_int32), ("decay", C.c_int32), ("tid", C.c_uint32),
-        ("idx0", C.c_uint64),
+        ("idx0", C.c_uint64), ("wf", C.c_void_p), ("gf", C.c_void_p),
     ]
 
 
@@ -159,17 +159,21 @@ def hparams(beta1, beta2, eps, clip_d, weight_decay, annealed: bool = False):
 
 def tensor_step(w_bits: np.ndarray, g_bits: np.ndarray, st: TensorState, tid: int, hp, step: int,
                 lr: float, seed: int, want_x: bool = False, idx0: int = 0):
-    """One oracle step of one tensor; `w_bits` (uint16) and the state update in place.
+    """One oracle step of one tensor; `w_bits` and the state update in place. Weights and
+    gradient are both bf16 bit patterns (uint16) or both fp32 (an fp32 tensor: the new
+    weight is x, no dither).
 
     Returns a dict with Rbar, sum of U^2, RMS and kappa, plus the fp32 pre-rounding
-    values `x` and the dithers `r` when `want_x`.
+    values `x` and the dithers `r` (0 for an fp32 tensor) when `want_x`.
     """
-    assert w_bits.dtype == np.uint16 and g_bits.dtype == np.uint16
+    f32 = w_bits.dtype == np.float32
+    assert (w_bits.dtype, g_bits.dtype) in ((np.uint16, np.uint16), (np.float32, np.float32))
     assert w_bits.flags.c_contiguous and g_bits.flags.c_contiguous
     numel = st.n * st.m
     assert w_bits.size == numel and g_bits.size == numel
-    T = _Tensor(_ptr(w_bits), _ptr(g_bits), _ptr(st.M), _ptr(st.v), _ptr(st.R), _ptr(st.C),
-                st.n, st.m, st.kind, st.momentum, st.decay, tid, idx0)
+    T = _Tensor(None if f32 else _ptr(w_bits), None if f32 else _ptr(g_bits), _ptr(st.M), _ptr(st.v), _ptr(st.R),
+                _ptr(st.C), st.n, st.m, st.kind, st.momentum, st.decay, tid, idx0,
+                _ptr(w_bits) if f32 else None, _ptr(g_bits) if f32 else None)
     x = np.empty(numel, np.float32) if want_x else None
     r = np.empty(numel, np.uint16) if want_x else None
     stats = np.zeros(4, np.float64)

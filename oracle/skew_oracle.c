@@ -21,8 +21,10 @@
  * Arithmetic: every step is evaluated in double precision (built without
  * floating-point contraction, so x86 and Arm hosts agree bit for bit); state is
  * stored as fp32 (the memory model counts 4 bytes per state element); weights
- * and gradients are bf16 bit patterns. Each stored fp32 value is the
- * round-to-nearest-even conversion of the fp64 expression.
+ * and gradients are bf16 bit patterns, or fp32 for tensors kept in fp32 (App. A:
+ * "fp32 norms and router"), whose new weight is the fp32 value x itself with no
+ * dithered cast. Each stored fp32 value is the round-to-nearest-even conversion
+ * of the fp64 expression.
  *
  * Readings taken where the paper is silent or loose (each is listed in the
  * design notes with its reason):
@@ -233,7 +235,15 @@ typedef struct {
     uint32_t tid;       /* tensor id fed to the dither                           */
     uint64_t idx0;      /* dither index of element 0: 0, or for matrix e of a    */
                         /* stacked (E, n, m) tensor e*n*m (its flat offset)      */
+    float *wf;          /* fp32 tensor: weights (then w and g are unused), or NULL */
+    const float *gf;    /* fp32 tensor: gradient                                 */
 } so_tensor_t;
+
+/* Gradient element e as a double (bf16 bits or fp32). */
+static double so_grad(const so_tensor_t *T, int64_t e)
+{
+    return T->gf ? (double)T->gf[e] : so_bf16_to_double(T->g[e]);
+}
 
 typedef struct {
     double beta1, beta2, eps, clip_d, weight_decay;
@@ -270,7 +280,7 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
     /* Second moment: full (Algorithm 1, full branch) or factored (Eq. 1). */
     if (T->kind == SO_KIND_FULL) {
         for (int64_t e = 0; e < numel; ++e) {
-            double g = so_bf16_to_double(T->g[e]);
+            double g = so_grad(T, e);
             T->v[e] = (float)(b2 * (double)T->v[e] + (1.0 - b2) * g * g);
         }
     } else {
@@ -279,7 +289,7 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
         if (!rs || !cs) { free(rs); free(cs); free(U); return -1; }
         for (int64_t i = 0; i < n; ++i)
             for (int64_t j = 0; j < m; ++j) {
-                double g = so_bf16_to_double(T->g[i * m + j]);
+                double g = so_grad(T, i * m + j);
                 rs[i] += g * g;
                 cs[j] += g * g;
             }
@@ -298,7 +308,7 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
     for (int64_t i = 0; i < n; ++i)
         for (int64_t j = 0; j < m; ++j) {
             const int64_t e = i * m + j;
-            double g = so_bf16_to_double(T->g[e]);
+            double g = so_grad(T, e);
             double vhat;
             if (T->kind == SO_KIND_FULL)
                 vhat = (double)T->v[e];
@@ -319,13 +329,19 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
     const double rho = sqrt(su2 / (double)numel);
     const double kappa = 1.0 / fmax(1.0, rho / hp->clip_d);
 
-    /* Decoupled weight decay fused ahead of the dithered bf16 cast. */
+    /* Decoupled weight decay fused ahead of the dithered bf16 cast (an fp32
+     * tensor stores x itself). */
     const double lam = T->decay ? hp->weight_decay : 0.0;
     for (int64_t e = 0; e < numel; ++e) {
-        double w = so_bf16_to_double(T->w[e]);
+        double w = T->wf ? (double)T->wf[e] : so_bf16_to_double(T->w[e]);
         float x = (float)(w * (1.0 - lr * lam) - lr * kappa * U[e]);
-        uint16_t r = so_dither16(seed, t, T->tid, T->idx0 + (uint64_t)e);
-        T->w[e] = so_sr_bf16(x, r);
+        uint16_t r = 0;
+        if (T->wf) {
+            T->wf[e] = x;
+        } else {
+            r = so_dither16(seed, t, T->tid, T->idx0 + (uint64_t)e);
+            T->w[e] = so_sr_bf16(x, r);
+        }
         if (x_out) x_out[e] = x;
         if (r_out) r_out[e] = r;
     }

@@ -35,6 +35,7 @@ struct TPlan {
     int64_t moff = -1, voff = -1, roff = -1, coff = -1;  // floats into the state
     uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
     uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0;
+    uint32_t f32 = 0;         // SKEW_F_FP32: fp32 weights and gradient
     // bytes into the workspace
     size_t ws_rowp = 0, ws_colp = 0, ws_bsc = 0, ws_rsum = 0, ws_u2 = 0, ws_pp = 0, ws_rmin = 0, ws_fsum = 0, ws_fmin = 0;
 };
@@ -151,7 +152,8 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
         if (((uintptr_t)d.weight & 1) || ((uintptr_t)d.grad & 1)) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: bf16 pointers must be 2-byte aligned", k); }
         if (d.ndim < 1 || d.ndim > 3) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: ndim must be 1, 2 or 3", k); }
         if (d.tier < SKEW_TIER_BACKBONE || d.tier > SKEW_TIER_ROUTER) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: unknown tier %d", k, d.tier); }
-        if (d.flags & ~SKEW_F_NO_DECAY) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: unknown flags", k); }
+        if (d.flags & ~(SKEW_F_NO_DECAY | SKEW_F_FP32)) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: unknown flags", k); }
+        if ((d.flags & SKEW_F_FP32) && (((uintptr_t)d.weight | (uintptr_t)d.grad) & 3)) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: fp32 pointers must be 4-byte aligned", k); }
         if (d.ndim == 3 ? d.stack < 1 : d.stack != 0) { delete h; return fail(nullptr, SKEW_EINVAL, "tensor %d: stack must be >= 1 when ndim == 3 and 0 otherwise", k); }
         const int64_t E = d.ndim == 3 ? (int64_t)d.stack : 1;
         p.n = d.shape[0];
@@ -167,13 +169,16 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
         try {
             h->first[k] = (uint32_t)h->t.size();
             h->count[k] = (uint32_t)E;
+            const int64_t esize = (d.flags & SKEW_F_FP32) ? 4 : 2;  // bytes per weight / gradient element
             for (int64_t e = 0; e < E; ++e) {
                 TPlan q = p;
-                q.w = (uint16_t *)d.weight + e * p.numel;
-                q.g = (const uint16_t *)d.grad + e * p.numel;
+                q.w = (char *)d.weight + e * p.numel * esize;
+                q.g = (const char *)d.grad + e * p.numel * esize;
                 q.tid = (uint32_t)k;
                 q.base = (uint64_t)(e * p.numel);
-                geometry(q, (((uintptr_t)q.w | (uintptr_t)q.g) & 15) == 0);
+                q.f32 = (d.flags & SKEW_F_FP32) ? 1u : 0u;
+                // whole-row tiles and 16-byte vectors are for bf16 rows
+                geometry(q, !q.f32 && (((uintptr_t)q.w | (uintptr_t)q.g) & 15) == 0);
                 h->n_rowpath += q.rowpath;
                 h->t.push_back(q);
             }
@@ -357,13 +362,14 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.kind = p.kind;
         T.momentum = p.momentum;
         T.decay = p.decay;
-        bool vec = al16(T.w) && al16(T.g) && (!T.M || al16(T.M));
+        bool vec = !p.f32 && al16(T.w) && al16(T.g) && (!T.M || al16(T.M));
         if (p.kind == kKindFull)
             vec = vec && (p.numel % 8 == 0) && al16(T.v);
         else
             vec = vec && (p.m % 8 == 0);
         p.vec = vec ? 1 : 0;
         T.vec = p.vec;
+        T.f32 = p.f32;
         T.lcl = p.lcl;
         T.strips = p.strips;
         T.rowtiles = p.rowtiles;

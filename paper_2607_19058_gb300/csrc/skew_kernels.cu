@@ -99,6 +99,19 @@ __device__ __forceinline__ void load_bf8_scalar(const uint16_t *p, int valid, fl
     for (int c = 0; c < 8; ++c) o[c] = c < valid ? bf16_to_f32(p[c]) : 0.f;
 }
 
+// Elements e0 .. e0+7 of a weight or gradient array on the scalar path (elements
+// >= valid read as 0): bf16, or fp32 for a tensor kept in fp32 (its array pointer
+// then addresses floats).
+__device__ __forceinline__ void load8_elem(const uint16_t *base, bool f32, int64_t e0, int valid, float (&o)[8]) {
+    if (f32) {
+        const float *p = reinterpret_cast<const float *>(base) + e0;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) o[c] = c < valid ? p[c] : 0.f;
+    } else {
+        load_bf8_scalar(base + e0, valid, o);
+    }
+}
+
 // Eight fp32 values; `cg` reads through L2 only (values an earlier phase wrote).
 template <bool VEC>
 __device__ __forceinline__ void load_f8(const float *p, int valid, float (&o)[8], bool cg) {
@@ -469,7 +482,7 @@ __device__ void sumsq_tile(const TensorDev &T, uint32_t tile, Smem &sm, const Po
             const int64_t i = row0 + k * RG;
             float g[8];
             if (act && i < n)
-                load_bf8_scalar(g_ + i * m + col0, F.valid, g);
+                load8_elem(g_, T.f32, i * m + col0, F.valid, g);
             else
 #pragma unroll
                 for (int c = 0; c < 8; ++c) g[c] = 0.f;
@@ -1077,7 +1090,7 @@ __device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
             const int64_t i = row0 + k * RG;
             if (i >= n) break;
             float y[8];
-            load_bf8_scalar(g_ + i * m + col0, valid, y);
+            load8_elem(g_, T.f32, i * m + col0, valid, y);
             if (MOM) {
                 float mm[8];
                 load_f8<false>(M_ + i * m + col0, valid, mm, false);
@@ -1102,7 +1115,7 @@ __device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
         if (VEC)
             unpack_bf8(ld16_hint(T.g + e0, pol.drop), g);
         else
-            load_bf8_scalar(T.g + e0, valid, g);
+            load8_elem(T.g, T.f32, e0, valid, g);
         load_f8<VEC>(T.v + e0, valid, v, false);
 #pragma unroll
         for (int c = 0; c < 8; ++c) v[c] = fmaf(A.b2, v[c], A.c2 * (g[c] * g[c]));
@@ -1192,6 +1205,20 @@ __device__ __forceinline__ void write8(uint16_t *__restrict__ w, const Dith &d, 
     }
 }
 
+// Scalar-path write-back of elements e0 .. e0+valid-1: the dithered bf16 rounding,
+// or for a tensor kept in fp32 the fp32 value x itself.
+__device__ __forceinline__ void store8_elem(const TensorDev &T, uint16_t *w, const Dith &d, int64_t e0, int valid,
+                                            const float (&x)[8], const Pol &pol) {
+    if (T.f32) {
+        float *p = reinterpret_cast<float *>(w) + e0;
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+            if (c < valid) p[c] = x[c];
+    } else {
+        write8<false>(w, d, e0, valid, ((e0 + d.base) & 7) == 0, x, pol);
+    }
+}
+
 // FAST: no element of the tile reaches the clamp (fill_meta), so the update is
 // (-lr*kappa*coef * a_i) * b_j * y, one multiply and one fma per element.
 template <bool VEC, bool MOM, bool FAST>
@@ -1274,12 +1301,12 @@ __device__ void apply_fact_tile(const StepArgs &A, const TensorDev &T, const Ten
             if (MOM)
                 load_f8<false>(M_ + e0, valid, y, true);
             else
-                load_bf8_scalar(g_ + e0, valid, y);
-            load_bf8_scalar(w_ + e0, valid, w);
+                load8_elem(g_, T.f32, e0, valid, y);
+            load8_elem(w_, T.f32, e0, valid, w);
             const float a = rows[k * RG];
 #pragma unroll
             for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(a * b[c], ce), w[c] * wdf);
-            write8<false>(w_, d, e0, valid, ((e0 + d.base) & 7) == 0, x, pol);
+            store8_elem(T, w_, d, e0, valid, x, pol);
         }
     }
 }
@@ -1299,16 +1326,19 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
         else if (VEC)
             unpack_bf8(ld16_hint(T.g + e0, pol.drop), y);
         else
-            load_bf8_scalar(T.g + e0, valid, y);
+            load8_elem(T.g, T.f32, e0, valid, y);
         load_f8<VEC>(T.v + e0, valid, v, true);
         if (VEC)
             unpack_bf8(ld16_hint(T.w + e0, pol.drop), w);
         else
-            load_bf8_scalar(T.w + e0, valid, w);
+            load8_elem(T.w, T.f32, e0, valid, w);
 #pragma unroll
         for (int c = 0; c < 8; ++c) x[c] = fmaf(-coefC, y[c] * fminf(__frsqrt_rn(v[c]), A.ce), w[c] * wdf);
         const Dith dd = dith_of(A, T);  // on the vector path e0 and base are multiples of 8
-        write8<VEC>(T.w, dd, e0, valid, VEC || ((e0 + dd.base) & 7) == 0, x, pol);
+        if (VEC)
+            write8<true>(T.w, dd, e0, valid, true, x, pol);
+        else
+            store8_elem(T, T.w, dd, e0, valid, x, pol);
     }
 }
 

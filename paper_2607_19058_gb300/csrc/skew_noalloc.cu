@@ -81,7 +81,9 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     if (((uintptr_t)state & 3)) return SKEW_EINVAL;
     if (ndim != 1 && ndim != 2) return SKEW_EINVAL;
     if (tier < SKEW_TIER_BACKBONE || tier > SKEW_TIER_ROUTER) return SKEW_EINVAL;
-    if (flags & ~SKEW_F_NO_DECAY) return SKEW_EINVAL;
+    if (flags & ~(SKEW_F_NO_DECAY | SKEW_F_FP32)) return SKEW_EINVAL;
+    const bool f32 = (flags & SKEW_F_FP32) != 0;
+    if (f32 && (((uintptr_t)weight | (uintptr_t)grad) & 3)) return SKEW_EINVAL;
     const skew_hparams_t H = *hp;
     if (!std::isfinite(H.beta1) || H.beta1 < 0.f || H.beta1 >= 1.f) return SKEW_EINVAL;
     if (!std::isfinite(H.beta2) || H.beta2 < 0.f || H.beta2 >= 1.f) return SKEW_EINVAL;
@@ -111,7 +113,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     float *Cc = kind == kKindFactored ? after_m + n : nullptr;
 
     // ---- tile geometry and item counts (the planner's, plan_geometry) ---------------
-    const bool wg_aligned = (((uintptr_t)weight | (uintptr_t)grad) & 15) == 0;
+    const bool wg_aligned = !f32 && (((uintptr_t)weight | (uintptr_t)grad) & 15) == 0;  // row tiles: bf16 only
     const int64_t tiles64 = kind == kKindFactored ? ((m + 255) / 256) * ((n + 255) / 256)
                                                   : (numel + kFlatTileElems - 1) / kFlatTileElems;
     if (tiles64 > (int64_t(1) << 31)) return SKEW_EINVAL;
@@ -190,9 +192,10 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     td.momentum = momentum;
     td.decay = decay;
     auto al16 = [](const void *p) { return ((uintptr_t)p & 15) == 0; };
-    bool vec = al16(td.w) && al16(td.g) && (!td.M || al16(td.M));
+    bool vec = !f32 && al16(td.w) && al16(td.g) && (!td.M || al16(td.M));
     vec = kind == kKindFull ? (vec && numel % 8 == 0 && al16(td.v)) : (vec && m % 8 == 0);
     td.vec = vec ? 1 : 0;
+    td.f32 = f32 ? 1u : 0u;
     td.lcl = G.lcl;
     td.strips = G.strips;
     td.rowtiles = G.rowtiles;

@@ -140,7 +140,8 @@ struct TensorDev {
     uint32_t tid;       // dither tensor id
     uint64_t base;      // dither index of element 0 (a matrix of a stacked tensor: its offset)
     uint32_t kind, momentum, decay;
-    uint32_t vec;       // 1: 16-byte vector loads / stores are legal
+    uint32_t vec;       // 1: 16-byte vector loads / stores are legal (bf16 tensors only)
+    uint32_t f32;       // 1: weights and gradient are fp32 (w, g then address floats; no dither)
     uint32_t lcl;       // factored: log2 of lanes along a row (LC)
     uint32_t strips;    // factored: column strips of 8*LC columns
     uint32_t rowtiles;  // factored: row tiles of tile_rows rows; full: flat tiles

@@ -23,6 +23,7 @@ NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 TIER_BACKBONE, TIER_EXPERT, TIER_ROUTER = 0, 1, 2
 POLICY_TIERED, POLICY_EXPERT_MOMENTUM, POLICY_FACTORED_ROUTER, POLICY_UNIFORM, POLICY_ADAFACTOR = 0, 1, 2, 3, 4
 F_NO_DECAY = 1
+F_FP32 = 2
 KIND_FULL, KIND_FACTORED = 0, 1
 
 EXPORTS = ["skew_create", "skew_destroy", "skew_state_bytes", "skew_workspace_bytes", "skew_bind", "skew_step",
@@ -220,7 +221,9 @@ def hparams(beta1=0.9, beta2=0.999, eps=1e-8, clip_d=1.0, weight_decay=0.05, pol
 # torch convenience wrapper
 # --------------------------------------------------------------------------
 class SkewAdam:
-    """SkewAdam over a list of (weight, grad, tier[, flags]) bf16 CUDA tensors.
+    """SkewAdam over a list of (weight, grad, tier[, flags]) CUDA tensors, bf16 or fp32
+    (an fp32 pair, as the paper keeps the norms and the router, is stepped in fp32
+    with no dithered cast; F_FP32 is set for it).
 
     A 3-D tensor (E, n, m) is a stack of E matrices (e.g. an MoE layer's experts
     kept in one array), each stepped with its own second-moment factors and clip
@@ -236,8 +239,10 @@ class SkewAdam:
         for p in params:
             w, g, tier = p[0], p[1], p[2]
             flags = p[3] if len(p) > 3 else 0
-            if w.dtype != torch.bfloat16 or g.dtype != torch.bfloat16:
-                raise TypeError("weights and gradients must be bf16")
+            if w.dtype != g.dtype or w.dtype not in (torch.bfloat16, torch.float32):
+                raise TypeError("weights and gradients must both be bf16 or both fp32")
+            if w.dtype == torch.float32:
+                flags |= F_FP32
             if not (w.is_cuda and g.is_cuda and w.is_contiguous() and g.is_contiguous()):
                 raise ValueError("weights and gradients must be contiguous CUDA tensors")
             if w.shape != g.shape or w.dim() not in (1, 2, 3):

@@ -41,6 +41,11 @@ class Spec:
     tier: int
     expert: int = -1          # expert index for expert tensors
     no_decay: bool = False
+    fp32: bool = False        # weights and gradient kept in fp32 (App. A: norms and router)
+
+    @property
+    def dtype(self):
+        return torch.float32 if self.fp32 else torch.bfloat16
 
     @property
     def numel(self) -> int:
@@ -154,6 +159,22 @@ def ablation() -> Workload:
     return Workload("ablation", specs, HP(policy=POLICY_EXPERT_MOMENTUM), "normal", steps=20, n_experts=128)
 
 
+def toy_fp32() -> Workload:
+    """The toy set with the router and the norm vectors kept in fp32 (App. A)."""
+    wl = toy()
+    specs = [dataclasses.replace(s, fp32=True) if (s.tier == TIER_ROUTER or len(s.shape) == 1) else s
+             for s in wl.specs]
+    return dataclasses.replace(wl, name="toy_fp32", specs=specs)
+
+
+def appb_fp32() -> Workload:
+    """The App. B shapes at the paper's precision: router and LayerNorm vectors fp32 (App. A)."""
+    wl = appb()
+    specs = [dataclasses.replace(s, fp32=True) if (s.tier == TIER_ROUTER or len(s.shape) == 1) else s
+             for s in wl.specs]
+    return dataclasses.replace(wl, name="appb_fp32", specs=specs)
+
+
 def adafactor() -> Workload:
     """The App. B shapes under the Adafactor comparator (Sec. 5, App. A): every matrix
     factored, no momentum, beta2_t = 1 - t^-0.8."""
@@ -188,7 +209,7 @@ def stack_experts(wl: Workload) -> Workload:
 
 
 WORKLOADS = {"small": small, "toy": toy, "slice": slice_, "appb": appb, "literal": literal, "skewed": skewed,
-             "ablation": ablation, "adafactor": adafactor}
+             "ablation": ablation, "adafactor": adafactor, "toy_fp32": toy_fp32, "appb_fp32": appb_fp32}
 
 
 def get(name: str) -> Workload:
@@ -219,9 +240,9 @@ def _normal(shape, std, gen, device) -> torch.Tensor:
 
 
 def init_weight(wl: Workload, tid: int, device="cpu") -> torch.Tensor:
-    """W ~ N(0, 0.02^2), bf16."""
+    """W ~ N(0, 0.02^2), bf16 (fp32 for an fp32 tensor)."""
     s = wl.specs[tid]
-    return _normal(s.shape, 0.02, _gen(device, wl.seed, 1, tid), device).to(torch.bfloat16)
+    return _normal(s.shape, 0.02, _gen(device, wl.seed, 1, tid), device).to(s.dtype)
 
 
 def dirichlet_loads(n: int, seed: int) -> torch.Tensor:
@@ -248,29 +269,34 @@ def _student_t3(shape, gen, device) -> torch.Tensor:
 
 
 def grad(wl: Workload, tid: int, step: int, device="cpu") -> torch.Tensor:
-    """Gradient of tensor `tid` at (1-based) `step`, bf16, per the workload's recipe."""
+    """Gradient of tensor `tid` at (1-based) `step` per the workload's recipe, bf16 (fp32
+    for an fp32 tensor: the same fp32 draw, not rounded)."""
+    return _grad32(wl, tid, step, device).to(wl.specs[tid].dtype)
+
+
+def _grad32(wl: Workload, tid: int, step: int, device) -> torch.Tensor:
     s = wl.specs[tid]
     gen = _gen(device, wl.seed, 2, step, tid)
     if wl.grad_kind == "toy":
         if s.tier == TIER_EXPERT and s.expert in (5, 6, 7) and step % 2 == 1:
-            return torch.zeros(s.shape, dtype=torch.bfloat16, device=device)
-        return _normal(s.shape, 1e-3, gen, device).to(torch.bfloat16)
+            return torch.zeros(s.shape, dtype=torch.float32, device=device)
+        return _normal(s.shape, 1e-3, gen, device)
     if wl.grad_kind == "slice":
         if s.tier == TIER_EXPERT:
             load = float(dirichlet_loads(wl.n_experts, wl.seed)[s.expert])
-            return _normal(s.shape, 1e-3 * math.sqrt(64.0 * load), gen, device).to(torch.bfloat16)
-        return _normal(s.shape, 1e-3, gen, device).to(torch.bfloat16)
+            return _normal(s.shape, 1e-3 * math.sqrt(64.0 * load), gen, device)
+        return _normal(s.shape, 1e-3, gen, device)
     if wl.grad_kind == "skewed":
         if s.tier == TIER_EXPERT:
             rank = int(zipf_ranks(wl.n_experts, wl.seed, step)[s.expert])
             if rank > wl.n_experts - 40:      # the 40 least-loaded experts see no tokens
-                return torch.zeros(s.shape, dtype=torch.bfloat16, device=device)
-            return (1e-3 * _student_t3(s.shape, gen, device)).to(torch.bfloat16)
+                return torch.zeros(s.shape, dtype=torch.float32, device=device)
+            return (1e-3 * _student_t3(s.shape, gen, device))
         g = _normal(s.shape, 1e-3, gen, device)
         if s.tier == TIER_ROUTER and step % 10 == 7:
             g = g * 100.0
-        return g.to(torch.bfloat16)
-    return _normal(s.shape, 1e-3, gen, device).to(torch.bfloat16)
+        return g
+    return _normal(s.shape, 1e-3, gen, device)
 
 
 def bf16_bits(t: torch.Tensor):

@@ -47,6 +47,21 @@ def bits16(t: torch.Tensor) -> np.ndarray:
     return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16).reshape(-1).copy()
 
 
+def host_copy(t: torch.Tensor) -> np.ndarray:
+    """Host copy of a weight / gradient tensor as the oracle takes it: bf16 bit patterns, or
+    fp32 values for a tensor kept in fp32."""
+    if t.dtype == torch.float32:
+        return t.detach().contiguous().cpu().numpy().reshape(-1).copy()
+    return bits16(t)
+
+
+def as_f64(a: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns or fp32 values as float64."""
+    if a.dtype == np.uint16:
+        return (a.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return a.astype(np.float64)
+
+
 def f32(t: torch.Tensor) -> np.ndarray:
     return t.detach().float().cpu().numpy().reshape(-1).copy()
 
@@ -102,6 +117,31 @@ def rel_err_terms(a: np.ndarray, b: np.ndarray, scale: np.ndarray) -> float:
 
 def _bits_to_f64(b32: np.ndarray) -> np.ndarray:
     return np.asarray(b32, np.uint32).view(np.float32).astype(np.float64)
+
+
+def compare_weights_f32(gpu_w: np.ndarray, x: np.ndarray, w_pre: np.ndarray, wdf: float, where: str,
+                        upd_terms=None) -> (int, float):
+    """fp32 tensors (no dither): the GPU's weight is its fp32 evaluation of x; every element
+    must lie within X_RTOL * S of the oracle's x, S = |w (1 - lr lambda)| + the magnitude of
+    the update's terms, and non-finite values must match exactly."""
+    g64, x64 = gpu_w.astype(np.float64), x.astype(np.float64)
+    fin = np.isfinite(x64)
+    inf = np.isinf(x64)
+    assert np.array_equal(np.isnan(g64), np.isnan(x64)) and np.array_equal(g64[inf], x64[inf]), \
+        f"{where}: non-finite fp32 weights differ"
+    diff = (gpu_w.view(np.uint32) != x.view(np.uint32)) & fin
+    nbad = int(diff.sum())
+    worst = 0.0
+    if nbad:
+        t1 = w_pre[diff].astype(np.float64) * wdf
+        upd = np.abs(t1 - x64[diff])
+        if upd_terms is not None:
+            upd = np.maximum(upd, upd_terms(np.nonzero(diff)[0]))
+        S = np.abs(t1) + upd
+        rel = np.abs(g64[diff] - x64[diff]) / np.maximum(S, 1e-300)
+        worst = float(rel.max())
+        assert worst <= X_RTOL, f"{where}: fp32 weight {worst:.3e} S from the oracle's x"
+    return 0, worst
 
 
 def compare_weights(gpu_w: np.ndarray, ora_w: np.ndarray, x: np.ndarray, r: np.ndarray, w_pre: np.ndarray,
@@ -210,7 +250,7 @@ class Harness:
         pre = {}
         for k in self.check:   # teacher forcing: the oracle starts from the GPU's pre-step values
             gs = self._gpu_state(k)
-            wb, gb = bits16(self.W[k]), bits16(self.G[k])
+            wb, gb = host_copy(self.W[k]), host_copy(self.G[k])
             nm = wb.size // self._stack(k)
             pre[k] = {}
             for e, st in self.ostate[k].items():
@@ -223,7 +263,7 @@ class Harness:
         self.opt.sync_status()
         rep = Report()
         for k in self.check:
-            gws, gss = bits16(self.W[k]), self._gpu_state(k)
+            gws, gss = host_copy(self.W[k]), self._gpu_state(k)
             for e, st in self.ostate[k].items():
                 rep.merge(self._check_matrix(k, e, st, pre[k][e], gws, gss[e], t, seed))
         assert rep.w_mismatch <= W_MISMATCH_FRAC * rep.elements, \
@@ -241,12 +281,15 @@ class Harness:
         lam = float(np.float32(self.hpd["weight_decay"])) if st.decay else 0.0
         wdf = 1.0 - float(np.float32(self.lr)) * lam
         terms = self._momentum_update_terms(st, o, g, m_prev, t) if st.momentum else None
-        nbad, worst = compare_weights(gw, w0, o["x"], o["r"], wpre, wdf, where, terms)
+        if gw.dtype == np.float32:
+            nbad, worst = compare_weights_f32(gw, o["x"], wpre, wdf, where, terms)
+        else:
+            nbad, worst = compare_weights(gw, w0, o["x"], o["r"], wpre, wdf, where, terms)
         worst_state = 0.0
         for key in ("M", "v", "R", "C"):
             if getattr(st, key) is not None:
                 if key == "M":
-                    gd = (g.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+                    gd = as_f64(g)
                     b1 = float(np.float32(self.hpd["beta1"]))
                     scale = b1 * np.abs(m_prev.astype(np.float64)) + (1 - b1) * np.abs(gd)
                     err = rel_err_terms(gs[key], st.M, scale)
@@ -279,7 +322,7 @@ class Harness:
                 vhat = (st.R[i].astype(np.float64) * st.C[j].astype(np.float64) / o["rbar"]
                         if o["rbar"] > 0 else np.zeros(idx.size))
             inv = 1.0 / np.sqrt(np.maximum(vhat, eps))
-            gd = (g[idx].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+            gd = as_f64(g[idx])
             mterms = b1 * np.abs(m_prev[idx].astype(np.float64)) + (1 - b1) * np.abs(gd)
             return lr * o["kappa"] * coef * inv * mterms
         return fn

@@ -219,3 +219,17 @@ def test_64bit_extents_plan():
     assert i.numel == 65536 * 40000 > 2**31
     assert S.skew_state_bytes(h) == 4 * (65536 + 40000) + 4 * 2 * 3 * 2**30
     S.skew_destroy(h)
+
+
+def test_fp32_tensors_plan():
+    """SKEW_F_FP32 (App. A: fp32 norms and router): accepted for any tier, 4-byte alignment
+    required, never on the whole-row bf16 path; the state is the same closed form."""
+    h = S.skew_create([_one((4096, 4096), flags=S.F_FP32), _one((4096, 4096)), _one((4096,), flags=S.F_FP32,
+                                                                                    tier=S.TIER_BACKBONE)],
+                      S.hparams())
+    assert [S.skew_tensor_info(h, k).rowpath for k in range(3)] == [0, 1, 0]
+    assert S.skew_state_bytes(h) == 4 * (2 * (4096 + 4096) + 2 * 4096)
+    S.skew_destroy(h)
+    with pytest.raises(S.SkewError) as e:
+        S.skew_create([_one((8, 8), weight=0x1002, flags=S.F_FP32)], S.hparams())
+    assert e.value.code == S.SKEW_EINVAL and "4-byte" in str(e.value)

@@ -282,3 +282,32 @@ def test_adafactor_comparator():
     for t in range(1, 4):
         h.step(t, seed=11 * t)
     h.close()
+
+
+def test_fp32_router_and_norms():
+    """The paper's precision (App. A): router and LayerNorm vectors in fp32, stepped with no
+    dithered cast, beside bf16 matrices; over the toy steps and at the paper's hyper-parameters."""
+    h = _harness(WL.toy_fp32())
+    assert any(w.dtype == torch.float32 for w in h.W)
+    for t in range(1, 6):
+        h.step(t)
+    h.close()
+    h = _harness(WL.toy_fp32(), hp_override=dict(eps=1e-8, lr=3e-4, weight_decay=0.05))
+    for t in range(1, 4):
+        h.step(t, seed=5)
+    h.close()
+
+
+def test_fp32_awkward_shapes_and_policies():
+    """fp32 tensors on the strip path (factored, with and without momentum, ragged), flat
+    tiles with a ragged tail, a stack, and under the factored-router and Adafactor policies."""
+    B, E, R = WL.TIER_BACKBONE, WL.TIER_EXPERT, WL.TIER_ROUTER
+    specs = [WL.Spec("r300x127", (300, 127), R, fp32=True), WL.Spec("v1001", (1001,), B, fp32=True),
+             WL.Spec("b37x4096", (37, 4096), B, fp32=True), WL.Spec("e77x333", (77, 333), E, fp32=True),
+             WL.Spec("s3x21x40", (3, 21, 40), E, fp32=True), WL.Spec("e64x4096", (64, 4096), E)]
+    for policy in (WL.POLICY_TIERED, WL.POLICY_FACTORED_ROUTER, WL.POLICY_ADAFACTOR):
+        wl = WL.Workload("fp32_edge", specs, WL.HP(policy=policy), "normal", steps=3)
+        h = _harness(wl)
+        for t in range(1, 4):
+            h.step(t, seed=t + policy)
+        h.close()

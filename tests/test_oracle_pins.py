@@ -378,6 +378,40 @@ def test_step1_full_v_gives_sign():
         assert np.max(np.abs(o["x"].astype(np.float64) - want)) <= 4e-7 * lr + np.spacing(want).max()
 
 
+def test_fp32_tensor_step1_and_bf16_agreement():
+    """fp32 norms and router (App. A): the new weight is the fp32 x itself (no dithered cast).
+    Step 1 on an fp32 vector gives U = sign(g) (Algorithm 1, full v); on inputs that are
+    exactly bf16 values, an fp32 tensor and a bf16 tensor see the same x and state, and the
+    bf16 tensor's weight is the dithered rounding of that x."""
+    rng = np.random.default_rng(31)
+    n = 777
+    gb = _bf16(rng.normal(0, 1e-3, n).astype(np.float32))
+    gb[::9] = 0
+    wb = _bf16(rng.normal(0, 0.02, n).astype(np.float32))
+    lr = float(F32(1e-3))
+    gf, wf = _f(gb), _f(wb)  # fp32 copies of the same values
+    for tier, shape in ((O.TIER_BACKBONE, (n,)), (O.TIER_ROUTER, (7, 111))):
+        sf, sb = O.TensorState(shape, tier), O.TensorState(shape, tier)
+        w32, w16 = wf.copy(), wb.copy()
+        for t in (1, 2):
+            of = O.tensor_step(w32, gf, sf, 5, _hp(), t, lr, 8, want_x=True)
+            ob = O.tensor_step(w16, gb, sb, 5, _hp(), t, lr, 8, want_x=True)
+            assert np.array_equal(w32.view(np.uint32), of["x"].view(np.uint32))   # stored as is
+            assert not of["r"].any()
+            if t == 1:  # x of step 1 is the bf16 path's x (same inputs, same state)
+                assert np.array_equal(of["x"].view(np.uint32), ob["x"].view(np.uint32))
+                for key in ("M", "v", "R", "C"):
+                    if getattr(sf, key) is not None:
+                        assert np.array_equal(getattr(sf, key), getattr(sb, key))
+                assert np.array_equal(w16, O.sr_bf16(ob["x"], ob["r"]))
+                if tier == O.TIER_BACKBONE:  # Algorithm 1, full v at t = 1: U = sign(g)
+                    lam = float(F32(0.1))
+                    want = (wf.astype(np.float64) * (1 - lr * lam) - lr * np.sign(gf)).astype(np.float32)
+                    assert np.max(np.abs(of["x"].astype(np.float64) - want)) <= 4e-7 * lr + np.spacing(want).max()
+            w16 = _bf16(w32)  # keep both paths on the same weights for the next step
+            w32 = _f(w16).copy()
+
+
 def test_clip_closed_form():
     """Zero grad at t=1 then g at t=2 on the full path: RMS = sqrt(1+beta2), update = sign(g)."""
     rng = np.random.default_rng(8)

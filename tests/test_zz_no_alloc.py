@@ -68,3 +68,28 @@ def test_noalloc_rejects_oversized_tensor():
         S.skew_step_tensor_noalloc(w.data_ptr(), w.data_ptr(), 2, rows, cols, S.TIER_EXPERT, 0, hp, w.data_ptr(),
                                    nbytes, 0, 1, 1e-3, 0, torch.cuda.current_stream().cuda_stream)
     assert e.value.code == S.SKEW_ETOOBIG
+
+
+def test_noalloc_fp32_matches_regular_path():
+    """An fp32 tensor (SKEW_F_FP32) through the no-alloc entry point equals skew_step's result."""
+    dev = torch.device("cuda")
+    for shape, tier in (((300, 127), S.TIER_ROUTER), ((4097,), S.TIER_BACKBONE)):
+        torch.manual_seed(1)
+        w0 = torch.randn(shape, device=dev) * 0.02
+        g = torch.empty(shape, device=dev)
+        hp = S.hparams(0.9, 0.999, 1e-30, 1.0, 0.1, S.POLICY_TIERED)
+        w_ref, w_na = w0.clone(), w0.clone()
+        ref = S.SkewAdam([(w_ref, g, tier)], hp)
+        nbytes = ref.state_bytes
+        state = torch.zeros(nbytes // 4, dtype=torch.float32, device=dev)
+        stream = torch.cuda.current_stream().cuda_stream
+        for t in (1, 2):
+            g.copy_(torch.randn(shape, device=dev) * 1e-3)
+            ref.step(t, 1e-3, 5)
+            S.skew_step_tensor_noalloc(w_na.data_ptr(), g.data_ptr(), len(shape), shape[0],
+                                       shape[1] if len(shape) == 2 else 0, tier, S.F_FP32, hp, state.data_ptr(),
+                                       nbytes, 0, t, 1e-3, 5, stream)
+            torch.cuda.synchronize()
+            assert torch.equal(w_ref, w_na), f"fp32 weights differ at step {t}"
+            assert torch.equal(ref.state[:nbytes].view(torch.float32), state)
+        ref.close()
