@@ -236,7 +236,7 @@ int skew_tensor_info(const skew_handle_t *h, int32_t tid, skew_tensor_info_t *ou
 /*
  * Benchmark support: launch timing. After skew_profile_begin(h, n), each of the
  * next n calls of skew_step records a CUDA event before and after each timed
- * launch it makes on the step's stream (six grouped launches, named by
+ * launch it makes on the step's stream (seven grouped launches, named by
  * skew_kernel_name; a phase with no work times ~0; no extra
  * synchronisation). skew_profile_end(h, ms, cap, &steps, &launches)
  * synchronises, writes the durations in milliseconds row-major into
