@@ -51,7 +51,7 @@ def parse():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="appb", help="shape set (appb = the paper's 6.78B App. B shapes)")
     p.add_argument("--seed", type=int, default=20260207)
-    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--e2e-steps", type=int, default=6)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="target oracle time of the CPU baseline sample")
@@ -300,6 +300,20 @@ def job_rate(world, params_per_rank, ms):
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+def flat_views(wl, dev):
+    """One device buffer holding every tensor of the workload (bf16, or fp32 for an fp32
+    tensor) at 128-byte aligned offsets; returns it and the per-tensor views."""
+    import torch
+    offs, total = [], 0
+    for s in wl.specs:
+        total = (total + 127) // 128 * 128
+        offs.append(total)
+        total += s.numel * (4 if s.fp32 else 2)
+    buf = torch.empty(max(total, 1), dtype=torch.uint8, device=dev)
+    views = [buf[o:o + s.numel * (4 if s.fp32 else 2)].view(s.dtype).view(s.shape) for o, s in zip(offs, wl.specs)]
+    return buf, views
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -317,9 +331,13 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     wl = WL.get(args.workload)
     hp = wl.hp
-    # inputs resident in HBM before timing
-    W = [WL.init_weight(wl, k, dev) for k in range(len(wl.specs))]
-    G = [WL.grad(wl, k, 1, dev) for k in range(len(wl.specs))]
+    # inputs resident in HBM before timing: every weight (gradient) a 128-byte aligned view
+    # of one device buffer, so the end-to-end leg moves each direction in one copy
+    Wbuf, W = flat_views(wl, dev)
+    Gbuf, G = flat_views(wl, dev)
+    for k in range(len(wl.specs)):
+        W[k].copy_(WL.init_weight(wl, k, dev))
+        G[k].copy_(WL.grad(wl, k, 1, dev))
     params = [(W[k], G[k], s.tier, S.F_NO_DECAY if s.no_decay else 0) for k, s in enumerate(wl.specs)]
     opt = S.SkewAdam(params, S.hparams(hp.beta1, hp.beta2, hp.eps, hp.clip_d, hp.weight_decay, hp.policy))
     bm = byte_model(opt, len(wl.specs))
@@ -359,39 +377,51 @@ def run_ours(args):
     achieved = dom_bytes / (kmean[dom] * 1e-3) / 1e9
     step_gbs = bm["step_min"] / (ms * 1e-3) / 1e9
 
-    # end to end through the C ABI with host buffers
+    # end to end through the C ABI with host buffers: every step copies all gradients in
+    # from pinned host memory (one copy) and all updated weights back out (one copy); the
+    # copy-in of step t+1 runs on its own stream beside the copy-out of step t (each waits
+    # only for the step that frees its buffer)
     e2e = None
     if not args.no_e2e and args.e2e_steps > 0:
-        total = sum(w.numel() for w in W)
-        hg = torch.empty(total, dtype=torch.bfloat16, pin_memory=True)
-        hw = torch.empty(total, dtype=torch.bfloat16, pin_memory=True)
-        off = 0
-        views = []
-        for k in range(len(W)):
-            n = W[k].numel()
-            hg[off:off + n].copy_(G[k].reshape(-1))
-            views.append((hg[off:off + n].view(G[k].shape), hw[off:off + n].view(W[k].shape)))
-            off += n
+        hg = torch.empty(Gbuf.numel(), dtype=torch.uint8, pin_memory=True)
+        hw = torch.empty(Wbuf.numel(), dtype=torch.uint8, pin_memory=True)
+        hg.copy_(Gbuf)
+        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
+        ev = lambda: torch.cuda.Event(enable_timing=False)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
+        a.record(s_in)
+        stepped = drained = None
         for _ in range(args.e2e_steps):
             step += 1
-            for k in range(len(W)):
-                G[k].copy_(views[k][0], non_blocking=True)
+            if stepped is not None:
+                s_in.wait_event(stepped)       # the previous step has read its gradients
+            with torch.cuda.stream(s_in):
+                Gbuf.copy_(hg, non_blocking=True)
+            loaded = ev()
+            loaded.record(s_in)
+            stream.wait_event(loaded)
+            if drained is not None:
+                stream.wait_event(drained)     # the previous weights are back on the host
             opt.step(step, hp.lr, args.seed)
-            for k in range(len(W)):
-                views[k][1].copy_(W[k], non_blocking=True)
-        b.record(stream)
+            stepped = ev()
+            stepped.record(stream)
+            s_out.wait_event(stepped)
+            with torch.cuda.stream(s_out):
+                hw.copy_(Wbuf, non_blocking=True)
+            drained = ev()
+            drained.record(s_out)
+        b.record(s_out)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(a.elapsed_time(b) / args.e2e_steps, world, dev)
         e2e = {"value": job_rate(world, bm["N"], e2e_ms), "unit": "params/s", "ms_per_step": e2e_ms,
-               "h2d_bytes_per_step": 2 * bm["N"], "d2h_bytes_per_step": 2 * bm["N"],
-               "path": "skew_step via ctypes; gradients copied in from pinned host memory and weights read back "
-                       "to pinned host memory every step"}
-        del hg, hw, views
+               "h2d_bytes_per_step": int(Gbuf.numel()), "d2h_bytes_per_step": int(Wbuf.numel()),
+               "path": "skew_step via ctypes; every step copies all gradients in from pinned host memory and all "
+                       "updated weights back to pinned host memory, one copy per direction, the copy-in of the "
+                       "next step beside the copy-out of the last"}
+        del hg, hw
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
