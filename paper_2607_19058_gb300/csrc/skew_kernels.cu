@@ -680,12 +680,12 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const float b2 = A.b2, c2 = A.c2, inv_m = 1.0f / (float)(8 * V);  // m is a power of two: exact
-    // per column pair: sums of g^2 and the compensated (hi, lo) sum of g^2 / R_i
-    float2 cs[NV][4], ph[NV][4], pl[NV][4];
+    // per column pair: sums of g^2, the compensated (hi, lo) sum of g^2 / R_i and its open fp32 part
+    float2 cs[NV][4], ph[NV][4], pl[NV][4], t[NV][4];
 #pragma unroll
     for (int v = 0; v < NV; ++v)
 #pragma unroll
-        for (int q = 0; q < 4; ++q) cs[v][q] = ph[v][q] = pl[v][q] = make_float2(0.f, 0.f);
+        for (int q = 0; q < 4; ++q) cs[v][q] = ph[v][q] = pl[v][q] = t[v][q] = make_float2(0.f, 0.f);
     double rsum = 0.0;                       // threads < CS: sum of the R of this chunk-row position
     float rmin = __int_as_float(0x7F800000);  // threads < CS: smallest positive R of it
     bool zero_row = false;
@@ -748,12 +748,8 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
             sm.inv[tid] = inv;
         }
         __syncthreads();
-        // pass 2: P_j += g^2 / R_i, a chunk sum per column folded into (hi, lo)
-        float2 t[NV][4];
-#pragma unroll
-        for (int v = 0; v < NV; ++v)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) t[v][q] = make_float2(0.f, 0.f);
+        // pass 2: P_j += g^2 / R_i, summed in fp32 over four chunks (at most 4 K rows)
+        // per column, then folded into (hi, lo)
 #pragma unroll
         for (int k = 0; k < K; ++k) {
             const int r = lay.rp + RPP * k;
@@ -769,15 +765,18 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
                 }
             }
         }
+        if ((c & 3u) == 3u || c + 1 == nch) {
 #pragma unroll
-        for (int v = 0; v < NV; ++v)
+            for (int v = 0; v < NV; ++v)
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                float2 s2, e2;
-                two_sum2(ph[v][q], t[v][q], s2, e2);
-                ph[v][q] = s2;
-                pl[v][q] = __fadd2_rn(pl[v][q], e2);
-            }
+                for (int q = 0; q < 4; ++q) {
+                    float2 s2, e2;
+                    two_sum2(ph[v][q], t[v][q], s2, e2);
+                    ph[v][q] = s2;
+                    pl[v][q] = __fadd2_rn(pl[v][q], e2);
+                    t[v][q] = make_float2(0.f, 0.f);
+                }
+        }
     }
     if (c < nch) {
         // A chunk did not land in time: record it, give the copies in flight
