@@ -302,11 +302,12 @@ def job_rate(world, params_per_rank, ms):
 # ---------------------------------------------------------------------------
 def flat_views(wl, dev):
     """One device buffer holding every tensor of the workload (bf16, or fp32 for an fp32
-    tensor) at 128-byte aligned offsets; returns it and the per-tensor views."""
+    tensor) at 512-byte aligned offsets (as the allocator places separate tensors);
+    returns it and the per-tensor views."""
     import torch
     offs, total = [], 0
     for s in wl.specs:
-        total = (total + 127) // 128 * 128
+        total = (total + 511) // 512 * 512
         offs.append(total)
         total += s.numel * (4 if s.fp32 else 2)
     buf = torch.empty(max(total, 1), dtype=torch.uint8, device=dev)
@@ -331,7 +332,7 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     wl = WL.get(args.workload)
     hp = wl.hp
-    # inputs resident in HBM before timing: every weight (gradient) a 128-byte aligned view
+    # inputs resident in HBM before timing: every weight (gradient) a 512-byte aligned view
     # of one device buffer, so the end-to-end leg moves each direction in one copy
     Wbuf, W = flat_views(wl, dev)
     Gbuf, G = flat_views(wl, dev)

@@ -711,10 +711,9 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
                     float2 g[4];
                     unpack_bf8x2(buf[r * V + v * TPB + lay.vi], g);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const float2 sq = __fmul2_rn(g[q], g[q]);
-                        cs[v][q] = __fadd2_rn(cs[v][q], sq);
-                        r2 = __fadd2_rn(r2, sq);
+                    for (int q = 0; q < 4; ++q) {  // g^2 into the column and row sums, one rounding each
+                        cs[v][q] = __ffma2_rn(g[q], g[q], cs[v][q]);
+                        r2 = __ffma2_rn(g[q], g[q], r2);
                     }
                 }
             }
