@@ -332,13 +332,10 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     wl = WL.get(args.workload)
     hp = wl.hp
-    # inputs resident in HBM before timing: every weight (gradient) a 512-byte aligned view
-    # of one device buffer, so the end-to-end leg moves each direction in one copy
-    Wbuf, W = flat_views(wl, dev)
-    Gbuf, G = flat_views(wl, dev)
-    for k in range(len(wl.specs)):
-        W[k].copy_(WL.init_weight(wl, k, dev))
-        G[k].copy_(WL.grad(wl, k, 1, dev))
+    # inputs resident in HBM before timing, one allocation per tensor (as a framework keeps
+    # its parameters)
+    W = [WL.init_weight(wl, k, dev) for k in range(len(wl.specs))]
+    G = [WL.grad(wl, k, 1, dev) for k in range(len(wl.specs))]
     params = [(W[k], G[k], s.tier, S.F_NO_DECAY if s.no_decay else 0) for k, s in enumerate(wl.specs)]
     opt = S.SkewAdam(params, S.hparams(hp.beta1, hp.beta2, hp.eps, hp.clip_d, hp.weight_decay, hp.policy))
     bm = byte_model(opt, len(wl.specs))
@@ -381,9 +378,22 @@ def run_ours(args):
     # end to end through the C ABI with host buffers: every step copies all gradients in
     # from pinned host memory (one copy) and all updated weights back out (one copy); the
     # copy-in of step t+1 runs on its own stream beside the copy-out of step t (each waits
-    # only for the step that frees its buffer)
+    # only for the step that frees its buffer). For one copy per direction this leg keeps
+    # every weight (gradient) as a 512-byte aligned view of one device buffer, in a handle
+    # of its own over the same parameters.
     e2e = None
     if not args.no_e2e and args.e2e_steps > 0:
+        Wbuf, Wf = flat_views(wl, dev)
+        Gbuf, Gf = flat_views(wl, dev)
+        for k in range(len(wl.specs)):
+            Wf[k].copy_(W[k])
+            Gf[k].copy_(G[k])
+        opt_e2e = S.SkewAdam([(Wf[k], Gf[k], s.tier, S.F_NO_DECAY if s.no_decay else 0)
+                              for k, s in enumerate(wl.specs)],
+                             S.hparams(hp.beta1, hp.beta2, hp.eps, hp.clip_d, hp.weight_decay, hp.policy))
+        for _ in range(args.warmup):
+            step += 1
+            opt_e2e.step(step, hp.lr, args.seed)
         hg = torch.empty(Gbuf.numel(), dtype=torch.uint8, pin_memory=True)
         hw = torch.empty(Wbuf.numel(), dtype=torch.uint8, pin_memory=True)
         hg.copy_(Gbuf)
@@ -406,7 +416,7 @@ def run_ours(args):
             stream.wait_event(loaded)
             if drained is not None:
                 stream.wait_event(drained)     # the previous weights are back on the host
-            opt.step(step, hp.lr, args.seed)
+            opt_e2e.step(step, hp.lr, args.seed)
             stepped = ev()
             stepped.record(stream)
             s_out.wait_event(stepped)
@@ -422,7 +432,9 @@ def run_ours(args):
                "path": "skew_step via ctypes; every step copies all gradients in from pinned host memory and all "
                        "updated weights back to pinned host memory, one copy per direction, the copy-in of the "
                        "next step beside the copy-out of the last"}
-        del hg, hw
+        opt_e2e.sync_status()
+        opt_e2e.close()
+        del hg, hw, Wf, Gf, Wbuf, Gbuf
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:

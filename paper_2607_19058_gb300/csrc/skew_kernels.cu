@@ -39,10 +39,10 @@ constexpr uint32_t kAll = 0xFFFFFFFFu;
 #define SKEW_MINB_SUMSQ 4
 #endif
 #ifndef SKEW_MINB_RMS
-#define SKEW_MINB_RMS 3
+#define SKEW_MINB_RMS 2
 #endif
 #ifndef SKEW_MINB_APPLY
-#define SKEW_MINB_APPLY 3
+#define SKEW_MINB_APPLY 2
 #endif
 constexpr int kSmemFloats = kVecPerThread * kThreads;  // row scales of the tallest tile
 constexpr int kStripCols = 8 * 32;                     // widest column strip
