@@ -121,7 +121,7 @@ def clocks_stop(handle):
 # ---------------------------------------------------------------------------
 def byte_model(opt, n_tensors):
     """Algorithmic minimum bytes of one step and of each kernel's own traffic."""
-    N = N_mom = N_full = N_fact = N_nomom = N_row = 0
+    N = N_mom = N_full = N_fact = N_nomom = N_row = N_rowm = 0
     rc = rc_row = 0
     for k in range(n_tensors):
         i = opt.info(k)
@@ -135,19 +135,21 @@ def byte_model(opt, n_tensors):
             N_full += i.numel
         elif i.rowpath:
             N_row += i.numel
+            N_rowm += i.numel if i.momentum else 0
             rc_row += E * (i.rows + i.cols)
         else:
             N_fact += i.numel
             rc += E * (i.rows + i.cols)
     step_min = 6 * N + 8 * N_mom + 8 * N_full + 8 * (rc + rc_row)
+    N_rest = N - N_row  # tensors of the strip / flat tiles
     kernels = {
         "k_sumsq": 2 * N_fact,                                   # read G of strip-path factored matrices
-        "k_rowsq": 2 * N_row + 8 * rc_row,                       # read G of row-path matrices; R read + write
+        "k_rowsq": 2 * N_row + 8 * N_rowm + 8 * rc_row,          # read G (and M r/w) of row-path matrices; R r/w
         "k_finalize": 8 * (rc + rc_row),                         # R, C read + write
-        "k_rms": 2 * (N - N_row) + 8 * N_mom + 8 * N_full,       # read G; M, v read + write
+        "k_rms": 2 * N_rest + 8 * (N_mom - N_rowm) + 8 * N_full,  # read G; M, v read + write
         "k_fallback": 0,                                          # runs only when a clamp may bind
-        "k_apply": 4 * (N - N_row) + 2 * (N_nomom - N_row) + 4 * N_mom + 4 * N_full,  # W r/w; G or M; v read
-        "k_apply_rows": 6 * N_row,                               # row path: W r/w, G read
+        "k_apply": 4 * N_rest + 2 * (N_nomom - (N_row - N_rowm)) + 4 * (N_mom - N_rowm) + 4 * N_full,
+        "k_apply_rows": 6 * N_row - 2 * N_rowm + 4 * N_rowm,     # W r/w and G (or the new M) read
     }
     return dict(N=N, N_mom=N_mom, N_full=N_full, rc=rc, step_min=step_min, kernels=kernels)
 

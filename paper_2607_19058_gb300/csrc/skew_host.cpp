@@ -34,7 +34,7 @@ struct TPlan {
     int64_t n = 0, m = 0, numel = 0;
     int64_t moff = -1, voff = -1, roff = -1, coff = -1;  // floats into the state
     uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
-    uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0;
+    uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0, fci = 0;
     uint32_t f32 = 0;         // SKEW_F_FP32: fp32 weights and gradient
     // bytes into the workspace
     size_t ws_rowp = 0, ws_colp = 0, ws_bsc = 0, ws_rsum = 0, ws_u2 = 0, ws_pp = 0, ws_rmin = 0, ws_fsum = 0, ws_fmin = 0;
@@ -114,6 +114,7 @@ static void geometry(TPlan &p, bool wg_aligned) {
     p.cr = g.cr;
     p.rt_rows = g.rt_rows;
     p.rtiles = g.rtiles;
+    p.fci = g.fci;
 }
 
 extern "C" {
@@ -381,6 +382,7 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.cr = p.cr;
         T.rt_rows = p.rt_rows;
         T.rtiles = p.rtiles;
+        T.fci = p.fci;
     }
     auto put = [&](size_t at, const std::vector<uint2> &v) {
         if (!v.empty()) std::memcpy(img.data() + (at - h->ws_tab), v.data(), v.size() * sizeof(uint2));

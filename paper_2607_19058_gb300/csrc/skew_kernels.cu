@@ -595,8 +595,8 @@ __device__ __forceinline__ RowChunk row_chunk(const TensorDev &T, uint32_t tile,
 }
 
 // Sum over a warp of K per-lane values, transposed: lane L ends with the total
-// of value j(L) (K = 8: j = 4*b4 + 2*b3 + b2 of L's bits; K = 4: j = 2*b4 + b3),
-// held by the lanes whose low bits (3 for K = 8, 2 + 1 for K = 4) are zero.
+// of value j(L) (K = 8: j = 4*b4 + 2*b3 + b2 of L's bits; K = 4: j = 2*b4 + b3;
+// K = 2: j = b4), held by the lanes whose low 2, 3 or 4 bits are zero.
 template <int K>
 __device__ __forceinline__ float warp_sum_transposed(const float (&x)[K], int &j) {
     const uint32_t ln = threadIdx.x & 31;
@@ -617,6 +617,14 @@ __device__ __forceinline__ float warp_sum_transposed(const float (&x)[K], int &j
         v1 += __shfl_xor_sync(kAll, v1, 2);
         v1 += __shfl_xor_sync(kAll, v1, 1);
         j = (b4 ? 4 : 0) + (b3 ? 2 : 0) + (b2 ? 1 : 0);
+        return v1;
+    } else if constexpr (K == 2) {
+        float v1 = (b4 ? x[1] : x[0]) + __shfl_xor_sync(kAll, b4 ? x[0] : x[1], 16);
+        v1 += __shfl_xor_sync(kAll, v1, 8);
+        v1 += __shfl_xor_sync(kAll, v1, 4);
+        v1 += __shfl_xor_sync(kAll, v1, 2);
+        v1 += __shfl_xor_sync(kAll, v1, 1);
+        j = b4 ? 1 : 0;
         return v1;
     } else {
         float v2[2];
@@ -900,31 +908,46 @@ __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem 
     const TensorDev &T = A.tensors[t];
     TensorScal &S = A.scal[t];
     const float inf = __int_as_float(0x7F800000);
-    const int64_t j = int64_t(local) * kFinChunk + threadIdx.x;
+    // the item's fci columns, kFinChunk / fci threads per column: thread tid adds the
+    // tiles r = sl, sl + tpc, ... of column cix (consecutive threads, consecutive columns)
+    const int fci = (int)T.fci, tpc = kFinChunk / fci;
+    const int cix = threadIdx.x % fci, sl = threadIdx.x / fci;
+    const int64_t j = int64_t(local) * fci + cix;
+    float cs = 0.f;  // this thread's tiles: sum of g^2 (in tile order) and, compensated, of g^2 / R_i
+    Acc2 pa;
+    if (j < T.m) {
+        const float2 *p = T.pp + j;
+        uint32_t r = sl;
+        for (; r + 15 * tpc < T.rtiles; r += 16 * tpc) {
+            float2 v[16];
+#pragma unroll
+            for (int q = 0; q < 16; ++q) v[q] = __ldcg(p + int64_t(r + q * tpc) * T.m);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+                cs += v[q].x;
+                pa.add(v[q].y);
+            }
+        }
+        for (; r < T.rtiles; r += tpc) {
+            const float2 v = __ldcg(p + int64_t(r) * T.m);
+            cs += v.x;
+            pa.add(v.y);
+        }
+    }
+    // the column's tpc parts in slice order
+    float *red = sm.colred;  // [3][kFinChunk]: sum g^2, hi, lo
+    red[threadIdx.x] = cs;
+    red[kFinChunk + threadIdx.x] = pa.hi;
+    red[2 * kFinChunk + threadIdx.x] = pa.lo;
+    __syncthreads();
     Acc2 contrib;
     float cmin = inf;
-    if (threadIdx.x < kFinChunk && j < T.m) {
+    if (sl == 0 && j < T.m) {
         const float Cold = __ldcg(T.C + j);
-        float cs = 0.f;  // sum over the row tiles of g^2 (in tile order) and, compensated, of g^2 / R_i
-        Acc2 pa;
-        {
-            const float2 *p = T.pp + j;
-            uint32_t r = 0;
-            for (; r + 16 <= T.rtiles; r += 16) {
-                float2 v[16];
-#pragma unroll
-                for (int q = 0; q < 16; ++q) v[q] = __ldcg(p + int64_t(r + q) * T.m);
-#pragma unroll
-                for (int q = 0; q < 16; ++q) {
-                    cs += v[q].x;
-                    pa.add(v[q].y);
-                }
-            }
-            for (; r < T.rtiles; ++r) {
-                const float2 v = __ldcg(p + int64_t(r) * T.m);
-                cs += v.x;
-                pa.add(v.y);
-            }
+        for (int k = 1; k < tpc; ++k) {
+            cs += red[k * fci + cix];
+            pa.add(red[kFinChunk + k * fci + cix]);
+            pa.lo += red[2 * kFinChunk + k * fci + cix];
         }
         const float P = pair_f(pa.hi, pa.lo);
         const float mean = __fdiv_rn(cs, (float)T.n);
@@ -944,6 +967,7 @@ __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem 
     }
 #pragma unroll
     for (int o = 16; o; o >>= 1) cmin = fminf(cmin, __shfl_xor_sync(kAll, cmin, o));
+    __syncthreads();  // the column parts in colred are consumed
     if ((threadIdx.x & 31) == 0) sm.colred[threadIdx.x >> 5] = cmin;
     const float2 cs2 = block_sum2(contrib, sm.red2);  // its barriers also publish colred
     if (threadIdx.x == 0) {
@@ -1045,6 +1069,7 @@ __device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
     const int64_t n = T.n, m = T.m, row0 = F.row0, RG = F.RG, col0 = F.col0;
     const int valid = F.valid;
     const float b1 = A.b1, c1 = A.c1, ce = A.ce;
+    const bool mnew = MOM && T.rowpath;  // phase B of a queued row-path tensor: M is already new
     const float *rows = meta.rows + F.rg;
     float b[8];
 #pragma unroll
@@ -1075,9 +1100,14 @@ __device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
                     if (MOM) {
                         const float4 m0 = mraw[MOM ? q : 0][0], m1 = mraw[MOM ? q : 0][1];
                         const float mm[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+                        if (mnew) {  // the row path already stored this step's momentum
 #pragma unroll
-                        for (int c = 0; c < 8; ++c) y[c] = fmaf(b1, mm[c], c1 * y[c]);
-                        store_f8<true>(M_ + i * m + col0, 8, y);
+                            for (int c = 0; c < 8; ++c) y[c] = mm[c];
+                        } else {
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) y[c] = fmaf(b1, mm[c], c1 * y[c]);
+                            store_f8<true>(M_ + i * m + col0, 8, y);
+                        }
                     }
                     rms_row(y, rows[(k0 + q) * RG], b, 8, ce, acc);
                 }
@@ -1092,9 +1122,14 @@ __device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
             if (MOM) {
                 float mm[8];
                 load_f8<false>(M_ + i * m + col0, valid, mm, false);
+                if (mnew) {
 #pragma unroll
-                for (int c = 0; c < 8; ++c) y[c] = fmaf(b1, mm[c], c1 * y[c]);
-                store_f8<false>(M_ + i * m + col0, valid, y);
+                    for (int c = 0; c < 8; ++c) y[c] = mm[c];
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) y[c] = fmaf(b1, mm[c], c1 * y[c]);
+                    store_f8<false>(M_ + i * m + col0, valid, y);
+                }
             }
             rms_row(y, rows[k * RG], b, valid, ce, acc);
         }
@@ -1500,6 +1535,375 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
 }
 
 // ---------------------------------------------------------------------------
+// Row path with momentum (backbone matrices, and experts under the momentum
+// variants). Phase A runs on whole rows as in k_rowsq and, in the same pass,
+// applies Algorithm 1's momentum update M <- b1 M + (1 - b1) g to a copy of the
+// rows of M made beside those of G, storing the new M. With U_ij = coef M_ij a_i b_j
+// and no element at the clamp, sum(U^2) = coef^2 * mean(R) * sum_j Q_j / C_j with
+// Q_j = sum_i M_ij^2 / R_i, accumulated here where the momentum-free path
+// accumulates P_j. Phase C then reads the new M where it would read G. A chunk
+// is CS = kMomGBytes / (2 m) rows: 16 KB of G (or W in phase C) and the same rows
+// of M (32 KB) in one slot of a 2-slot ring, one bulk copy each. A row whose R_i
+// is 0 or not finite sends the tensor to phase B (its momentum may still be
+// nonzero), where M is used as already updated.
+// ---------------------------------------------------------------------------
+constexpr int kMomStages = 2;
+constexpr int kMomSlot16 = 3 * kMomGBytes / 16;  // 16-byte words per slot: 16 KB bf16 | 32 KB fp32
+
+struct MomRowSmem {
+    uint4 buf[kMomStages][kMomSlot16];  // [G rows | M rows] per slot
+    uint64_t full[kMomStages];
+    float part[kRowThreads / 32][8];
+    float inv[32];
+    int fail;
+};
+
+// Issues the bulk copies of chunk c of row tile `tile` (rows of x = G in phase A,
+// W in phase C, and the same rows of M) into ring slot c % kMomStages.
+__device__ __forceinline__ void mom_issue(const TensorDev &T, const uint16_t *x, uint32_t tile, uint32_t c,
+                                          uint4 (*buf)[kMomSlot16], uint64_t *full, uint64_t pol) {
+    const RowChunk ch = row_chunk(T, tile, c);
+    const uint32_t bx = ch.rows * (uint32_t)T.m * 2u;
+    const int st = c % kMomStages;
+    mbar_expect_tx(&full[st], 3u * bx);
+    bulk_g2s(buf[st], x + ch.i0 * T.m, bx, &full[st], pol);
+    bulk_g2s(buf[st] + kMomGBytes / 16, T.M + ch.i0 * T.m, 2u * bx, &full[st], pol);
+}
+
+// k_rowsq for momentum tensors on TPB threads, rows of m = 8 V: chunks of CS = 1024 / V
+// rows, K = CS / RPP rows per thread per chunk.
+template <int TPB, int V>
+__device__ void rowsq_mom_tile(const StepArgs &A, const TensorDev &T, TensorScal &S, uint32_t tile, MomRowSmem &sm) {
+    using L = RowLayout<TPB, V>;
+    constexpr int NV = L::NV, RPP = L::RPP, WPR = L::WPR;
+    constexpr int CS = 1024 / V;
+    constexpr int K = CS / RPP;
+    static_assert(K == 2 || K == 4, "rows per thread per chunk");
+    const L lay;
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    const uint32_t nch = (uint32_t)min((int64_t)kMomChunks, (T.n - int64_t(tile) * T.rt_rows + T.cr - 1) / T.cr);
+    if (threadIdx.x == 0) {
+        for (int st = 0; st < kMomStages; ++st) mbar_init(&sm.full[st], 1);
+        fence_mbar_init();
+        sm.fail = 0;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+        for (uint32_t c = 0; c < nch && c < (uint32_t)kMomStages; ++c) mom_issue(T, T.g, tile, c, sm.buf, sm.full, pol);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const float b1 = A.b1, c1 = A.c1, b2 = A.b2, c2 = A.c2, inv_m = 1.0f / (float)(8 * V);  // exact
+    const float2 b12 = make_float2(b1, b1), c12 = make_float2(c1, c1);
+    // per column pair: sums of g^2, the compensated (hi, lo) sum of M^2 / R_i and its open fp32 part
+    float2 cs[NV][4], ph[NV][4], pl[NV][4], t[NV][4];
+#pragma unroll
+    for (int v = 0; v < NV; ++v)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) cs[v][q] = ph[v][q] = pl[v][q] = t[v][q] = make_float2(0.f, 0.f);
+    double rsum = 0.0;
+    float rmin = __int_as_float(0x7F800000);
+    bool zero_row = false;
+
+    uint32_t c = 0;
+    for (; c < nch; ++c) {
+        const int st = c % kMomStages;
+        const uint32_t par = (c / kMomStages) & 1u;
+        const RowChunk ch = row_chunk(T, tile, c);
+        float rp = 0.f;
+        if (tid < (int)ch.rows) rp = __ldcg(T.R + ch.i0 + tid);
+        const bool ok = mbar_wait(&sm.full[st], par);
+        const uint4 *bg = sm.buf[st];
+        const float4 *bm = reinterpret_cast<const float4 *>(sm.buf[st] + kMomGBytes / 16);
+        // pass 1: row sums and column sums of g^2
+        float rs[K];
+#pragma unroll
+        for (int k = 0; k < K; ++k) {
+            const int r = lay.rp + RPP * k;
+            float2 r2 = make_float2(0.f, 0.f);
+            if (r < (int)ch.rows) {
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    float2 g[4];
+                    unpack_bf8x2(bg[r * V + v * TPB + lay.vi], g);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        cs[v][q] = __ffma2_rn(g[q], g[q], cs[v][q]);
+                        r2 = __ffma2_rn(g[q], g[q], r2);
+                    }
+                }
+            }
+            rs[k] = r2.x + r2.y;
+        }
+        int j;
+        const float tot = warp_sum_transposed<K>(rs, j);
+        if ((lane & (K == 4 ? 7 : 15)) == 0) sm.part[warp][j] = tot;
+        if (__syncthreads_or(!ok)) break;  // every slot before this one has landed
+        if (tid == 0 && c >= 1 && c - 1 + kMomStages < nch) {
+            fence_proxy_async_smem();
+            mom_issue(T, T.g, tile, c - 1 + kMomStages, sm.buf, sm.full, pol);
+        }
+        if (tid < (int)ch.rows) {
+            const int w0 = (tid % RPP) * WPR, kr = tid / RPP;
+            float sum = 0.f;
+#pragma unroll
+            for (int w = 0; w < WPR; ++w) sum += sm.part[w0 + w][kr];
+            const float Rn = fmaf(b2, rp, c2 * (sum * inv_m));
+            T.R[ch.i0 + tid] = Rn;
+            rsum += (double)Rn;
+            float inv = 0.f;
+            if (Rn > 0.f && Rn < __int_as_float(0x7F800000)) {
+                rmin = fminf(rmin, Rn);
+                inv = __frcp_rn(Rn);
+            } else {
+                zero_row = true;  // R_i == 0 or not finite: its momentum may still be nonzero
+            }
+            sm.inv[tid] = inv;
+        }
+        __syncthreads();
+        // pass 2: M <- b1 M + (1 - b1) g (stored), Q_j += M^2 / R_i
+#pragma unroll
+        for (int k = 0; k < K; ++k) {
+            const int r = lay.rp + RPP * k;
+            if (r < (int)ch.rows) {
+                const float iv = sm.inv[r];
+                const float2 iv2 = make_float2(iv, iv);
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    const int vec = v * TPB + lay.vi;
+                    float2 g[4];
+                    unpack_bf8x2(bg[r * V + vec], g);
+                    const float4 m0 = bm[2 * (r * V + vec)], m1 = bm[2 * (r * V + vec) + 1];
+                    const float2 mo[4] = {make_float2(m0.x, m0.y), make_float2(m0.z, m0.w), make_float2(m1.x, m1.y),
+                                          make_float2(m1.z, m1.w)};
+                    float2 mn[4];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        mn[q] = __ffma2_rn(b12, mo[q], __fmul2_rn(c12, g[q]));
+                        t[v][q] = __ffma2_rn(__fmul2_rn(mn[q], mn[q]), iv2, t[v][q]);
+                    }
+                    float4 *dst = reinterpret_cast<float4 *>(T.M + (ch.i0 + r) * T.m + 8 * vec);
+                    dst[0] = make_float4(mn[0].x, mn[0].y, mn[1].x, mn[1].y);
+                    dst[1] = make_float4(mn[2].x, mn[2].y, mn[3].x, mn[3].y);
+                }
+            }
+        }
+        if ((c & 3u) == 3u || c + 1 == nch) {
+#pragma unroll
+            for (int v = 0; v < NV; ++v)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float2 s2, e2;
+                    two_sum2(ph[v][q], t[v][q], s2, e2);
+                    ph[v][q] = s2;
+                    pl[v][q] = __fadd2_rn(pl[v][q], e2);
+                    t[v][q] = make_float2(0.f, 0.f);
+                }
+        }
+    }
+    if (c < nch) {
+        // a chunk did not land in time: as in rowsq_tile
+        if (tid == 0) {
+            atomicOr(A.err, 2u);
+            const uint32_t issued_end = min(nch, c == 0 ? (uint32_t)kMomStages : c + kMomStages - 1);
+            for (uint32_t k = c; k < issued_end; ++k) (void)mbar_wait(&sm.full[k % kMomStages], (k / kMomStages) & 1u);
+        }
+        return;
+    }
+    const int64_t base = int64_t(tile) * 8 * V;
+    if constexpr (RPP == 1) {
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int64_t col = 8 * int64_t(v * TPB + lay.vi);
+            float4 *pp4 = reinterpret_cast<float4 *>(T.pp + base + col);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                pp4[q] = make_float4(cs[v][q].x, pair_f(ph[v][q].x, pl[v][q].x), cs[v][q].y,
+                                     pair_f(ph[v][q].y, pl[v][q].y));
+        }
+    } else {
+        // the ring is free (every chunk consumed before the last barrier): stage there
+        float *mcs = reinterpret_cast<float *>(sm.buf[0]);    // [TPB][8]
+        float2 *mpp = reinterpret_cast<float2 *>(sm.buf[1]);  // [TPB][8] (hi, lo)
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            mcs[tid * 8 + 2 * q] = cs[0][q].x;
+            mcs[tid * 8 + 2 * q + 1] = cs[0][q].y;
+            mpp[tid * 8 + 2 * q] = make_float2(ph[0][q].x, pl[0][q].x);
+            mpp[tid * 8 + 2 * q + 1] = make_float2(ph[0][q].y, pl[0][q].y);
+        }
+        __syncthreads();
+        for (int e = tid; e < 8 * V; e += TPB) {  // column e = 8 vi + q
+            const int vi = e >> 3, q = e & 7;
+            float cc = 0.f;
+            Acc2 pq;
+#pragma unroll
+            for (int r = 0; r < RPP; ++r) {
+                cc += mcs[(r * V + vi) * 8 + q];
+                const float2 h = mpp[(r * V + vi) * 8 + q];
+                pq.add(h.x);
+                pq.lo += h.y;
+            }
+            T.pp[base + e] = make_float2(cc, pair_f(pq.hi, pq.lo));
+        }
+    }
+    if (zero_row) atomicOr(&S.zflag, 1u);
+    if (warp == 0) {  // CS <= 32: the chunk-row positions are lanes of warp 0
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            rsum += __shfl_xor_sync(kAll, rsum, o);
+            rmin = fminf(rmin, __shfl_xor_sync(kAll, rmin, o));
+        }
+        if (lane == 0) {
+            T.rsum[tile] = rsum;
+            T.rmin[tile] = rmin;
+        }
+    }
+}
+
+struct MomApplySmem {
+    uint4 buf[kMomStages][kMomSlot16];  // [W rows | M rows] per slot
+    uint64_t full[kMomStages];
+    float a[kRowChunks * 32];           // row scales a_i of the tile (rt_rows <= 1024)
+    float red[2 * kRowThreads / 32];
+};
+
+// Phase C of a momentum row tile: as apply_rows_body with y = the new M (Algorithm 1,
+// backbone branch: U = coef M / D).
+template <int TPB, int V, bool FAST>
+__device__ void apply_rows_mom_body(const StepArgs &A, const TensorDev &T, uint32_t tile,
+                                    const float (&b)[RowLayout<TPB, V>::NV][8], float coefC, MomApplySmem &sm,
+                                    uint32_t nch, uint64_t pol) {
+    using L = RowLayout<TPB, V>;
+    constexpr int NV = L::NV, RPP = L::RPP;
+    constexpr int CA = 1024 / V, KA = CA / RPP;
+    const L lay;
+    const int tid = threadIdx.x;
+    const int64_t m = 8 * V;
+    uint16_t *__restrict__ w_ = T.w;
+    const Dith d = dith_of(A, T);
+    const float wdf = T.decay ? A.wdf : 1.0f;
+    const float ce = A.ce;
+    const float2 wdf2 = make_float2(wdf, wdf);
+    const Pol sp;
+    for (uint32_t c = 0; c < nch; ++c) {
+        const int st = c % kMomStages;
+        const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * CA;
+        const int rows = (int)min((int64_t)CA, T.n - i0);
+        const bool ok = mbar_wait(&sm.full[st], (c / kMomStages) & 1u);
+        const uint4 *bw = sm.buf[st];
+        const float4 *bm = reinterpret_cast<const float4 *>(sm.buf[st] + kMomGBytes / 16);
+#pragma unroll
+        for (int k = 0; k < KA; ++k) {
+            const int r = lay.rp + RPP * k;
+            if (r < rows) {
+                const float a = sm.a[c * CA + r];
+                const float cr = -coefC * a;
+                const float2 cr2 = make_float2(cr, cr);
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    const int vec = v * TPB + lay.vi;
+                    float w[8], x[8];
+                    unpack_bf8(bw[r * V + vec], w);
+                    const float4 m0 = bm[2 * (r * V + vec)], m1 = bm[2 * (r * V + vec) + 1];
+                    const float y[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+                    if constexpr (FAST) {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const float2 xx =
+                                __ffma2_rn(__fmul2_rn(cr2, make_float2(b[v][2 * q], b[v][2 * q + 1])),
+                                           make_float2(y[2 * q], y[2 * q + 1]),
+                                           __fmul2_rn(make_float2(w[2 * q], w[2 * q + 1]), wdf2));
+                            x[2 * q] = xx.x;
+                            x[2 * q + 1] = xx.y;
+                        }
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) x[q] = fmaf(-coefC, y[q] * fminf(a * b[v][q], ce), w[q] * wdf);
+                    }
+                    write8<true>(w_, d, (i0 + r) * m + 8 * vec, 8, true, x, sp);
+                }
+            }
+        }
+        // every thread is done with slot st: refill it with chunk c + kMomStages
+        if (__syncthreads_or(!ok)) {
+            if (tid == 0) {
+                atomicOr(A.err, 2u);
+                const uint32_t issued_end = min(nch, c + kMomStages);
+                for (uint32_t k = c; k < issued_end; ++k)
+                    (void)mbar_wait(&sm.full[k % kMomStages], (k / kMomStages) & 1u);
+            }
+            return;
+        }
+        if (tid == 0 && c + kMomStages < nch) {
+            fence_proxy_async_smem();
+            mom_issue(T, T.w, tile, c + kMomStages, sm.buf, sm.full, pol);
+        }
+    }
+}
+
+template <int TPB, int V>
+__device__ void apply_rows_mom_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile,
+                                    MomApplySmem &sm) {
+    using L = RowLayout<TPB, V>;
+    constexpr int NV = L::NV;
+    const L lay;
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    const int64_t r0 = int64_t(tile) * T.rt_rows;
+    const uint32_t rows_t = (uint32_t)min((int64_t)T.rt_rows, T.n - r0);
+    const uint32_t nch = (rows_t + T.cr - 1) / T.cr;
+    if (threadIdx.x == 0) {
+        for (int st = 0; st < kMomStages; ++st) mbar_init(&sm.full[st], 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+        for (uint32_t c = 0; c < nch && c < (uint32_t)kMomStages; ++c) mom_issue(T, T.w, tile, c, sm.buf, sm.full, pol);
+    const float rbar_s = __ldcg(&S.rbar_s);
+    const int rbar_e = __ldcg(&S.rbar_e);
+    float ma = 0.f, mb = 0.f;
+    for (uint32_t r = threadIdx.x; r < rows_t; r += TPB) {
+        const float a = row_scale(__ldcg(T.R + r0 + r), rbar_s, rbar_e);
+        sm.a[r] = a;
+        ma = fmaxf(ma, nan_to_inf(a));
+    }
+    float b[NV][8];
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+        const float *p = T.bsc + 8 * (v * TPB + lay.vi);
+        const float4 b0 = __ldcg(reinterpret_cast<const float4 *>(p));
+        const float4 b1 = __ldcg(reinterpret_cast<const float4 *>(p + 4));
+        b[v][0] = b0.x; b[v][1] = b0.y; b[v][2] = b0.z; b[v][3] = b0.w;
+        b[v][4] = b1.x; b[v][5] = b1.y; b[v][6] = b1.z; b[v][7] = b1.w;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mb = fmaxf(mb, nan_to_inf(b[v][k]));
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        ma = fmaxf(ma, __shfl_xor_sync(kAll, ma, o));
+        mb = fmaxf(mb, __shfl_xor_sync(kAll, mb, o));
+    }
+    if ((threadIdx.x & 31) == 0) {
+        sm.red[threadIdx.x >> 5] = ma;
+        sm.red[TPB / 32 + (threadIdx.x >> 5)] = mb;
+    }
+    __syncthreads();
+    ma = mb = 0.f;
+#pragma unroll
+    for (int w = 0; w < TPB / 32; ++w) {
+        ma = fmaxf(ma, sm.red[w]);
+        mb = fmaxf(mb, sm.red[TPB / 32 + w]);
+    }
+    const float coefC = __ldcg(&S.coefC);
+    if (ma * mb <= A.ce)
+        apply_rows_mom_body<TPB, V, true>(A, T, tile, b, coefC, sm, nch, pol);
+    else
+        apply_rows_mom_body<TPB, V, false>(A, T, tile, b, coefC, sm, nch, pol);
+}
+
+// ---------------------------------------------------------------------------
 // Kernels: one tile / item per CTA. The per-step parameters are a kernel
 // parameter (constant bank), so the dither keys and step scalars are uniform
 // operands of every warp.
@@ -1524,6 +1928,16 @@ __global__ void __launch_bounds__(kRowThreads, 512 / kRowThreads)
     const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
     TensorScal &S = A.scal[it.x];
+    if (T.momentum) {
+        MomRowSmem &ms = *reinterpret_cast<MomRowSmem *>(dyn_smem);
+        switch (T.m) {
+            case 4096: rowsq_mom_tile<kRowThreads, 512>(A, T, S, it.y, ms); break;
+            case 2048: rowsq_mom_tile<kRowThreads, 256>(A, T, S, it.y, ms); break;
+            case 1024: rowsq_mom_tile<kRowThreads, 128>(A, T, S, it.y, ms); break;
+            default: rowsq_mom_tile<kRowThreads, 64>(A, T, S, it.y, ms); break;  // 512
+        }
+        return;
+    }
     switch (T.m) {
         case 4096: rowsq_tile<kRowThreads, 512>(A, T, S, it.y, sm); break;
         case 2048: rowsq_tile<kRowThreads, 256>(A, T, S, it.y, sm); break;
@@ -1540,6 +1954,16 @@ __global__ void __launch_bounds__(kRowThreads, 512 / kRowThreads)
     const uint2 it = items[blockIdx.x];
     const TensorDev &T = A.tensors[it.x];
     const TensorScal &S = A.scal[it.x];
+    if (T.momentum) {
+        MomApplySmem &ms = *reinterpret_cast<MomApplySmem *>(dyn_smem);
+        switch (T.m) {
+            case 4096: apply_rows_mom_tile<kRowThreads, 512>(A, T, S, it.y, ms); break;
+            case 2048: apply_rows_mom_tile<kRowThreads, 256>(A, T, S, it.y, ms); break;
+            case 1024: apply_rows_mom_tile<kRowThreads, 128>(A, T, S, it.y, ms); break;
+            default: apply_rows_mom_tile<kRowThreads, 64>(A, T, S, it.y, ms); break;  // 512
+        }
+        return;
+    }
     switch (T.m) {
         case 4096: apply_rows_tile<kRowThreads, 512>(A, T, S, it.y, sm); break;
         case 2048: apply_rows_tile<kRowThreads, 256>(A, T, S, it.y, sm); break;
@@ -1629,9 +2053,10 @@ int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *co
     if (L.nA) k_sumsq<<<L.nA, kThreads, 0, s>>>(A, L.itemsA);
     mark(1);
     if (L.nR) {
-        const cudaError_t e = cudaFuncSetAttribute(k_rowsq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(RowSmem));
+        constexpr size_t kSm = sizeof(RowSmem) > sizeof(MomRowSmem) ? sizeof(RowSmem) : sizeof(MomRowSmem);
+        const cudaError_t e = cudaFuncSetAttribute(k_rowsq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSm);
         if (e != cudaSuccess) return (int)e;
-        k_rowsq<<<L.nR, kRowThreads, sizeof(RowSmem), s>>>(A, L.itemsR);
+        k_rowsq<<<L.nR, kRowThreads, kSm, s>>>(A, L.itemsR);
     }
     mark(2);
     if (L.nF) k_finalize<<<L.nF, kThreads, 0, s>>>(A, L.itemsF);
@@ -1643,10 +2068,11 @@ int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *co
     if (L.nC) k_apply<<<L.nC, kThreads, 0, s>>>(A, L.itemsC);
     mark(6);
     if (L.nCR) {
-        const cudaError_t e =
-            cudaFuncSetAttribute(k_apply_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(ApplyRowSmem));
+        constexpr size_t kSm =
+            sizeof(ApplyRowSmem) > sizeof(MomApplySmem) ? sizeof(ApplyRowSmem) : sizeof(MomApplySmem);
+        const cudaError_t e = cudaFuncSetAttribute(k_apply_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSm);
         if (e != cudaSuccess) return (int)e;
-        k_apply_rows<<<L.nCR, kRowThreads, sizeof(ApplyRowSmem), s>>>(A, L.itemsCR);
+        k_apply_rows<<<L.nCR, kRowThreads, kSm, s>>>(A, L.itemsCR);
     }
     mark(7);
     return (int)cudaGetLastError();

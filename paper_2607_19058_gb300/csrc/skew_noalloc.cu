@@ -207,6 +207,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     td.cr = G.cr;
     td.rt_rows = G.rt_rows;
     td.rtiles = G.rtiles;
+    td.fci = G.fci;
 
     // ---- per-step scalars, as skew_step forms them ------------------------------------
     const StepCoefs k = step_coefs(H, step);

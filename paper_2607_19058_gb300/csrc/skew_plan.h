@@ -26,6 +26,10 @@ constexpr int kFinChunk = 256;  // rows / columns per finalize item
 constexpr int kRowChunkBytes = 32768;
 constexpr int kRowChunks = 32;
 constexpr int kRowStages = 3;
+// Momentum tensors on the row path: a chunk holds kMomGBytes of bf16 rows (G in
+// phase A, W in phase C) and the same rows of fp32 M; a row tile is kMomChunks chunks.
+constexpr int kMomGBytes = 16384;
+constexpr int kMomChunks = 64;
 
 enum Kind : uint32_t { kKindFull = 0, kKindFactored = 1 };
 
@@ -82,6 +86,7 @@ inline StepCoefs step_coefs(const skew_hparams_t &H, int64_t step) {
 struct TileGeom {
     uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
     uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0;
+    uint32_t fci = 0;  // row path: columns per finalize item (kFinChunk / fci threads per column)
 };
 
 // `kind`, `momentum` as resolved by the tier policy; `wg_aligned`: weight and
@@ -101,14 +106,19 @@ inline TileGeom plan_geometry(uint32_t kind, uint32_t momentum, bool wg_aligned,
         g.rowtiles = (uint32_t)((n + g.tile_rows - 1) / g.tile_rows);
         g.ntiles = g.strips * g.rowtiles;
         g.nfc = (uint32_t)((m + kFinChunk - 1) / kFinChunk);
-        // Whole-row phases A and C: momentum-free factored matrices of width
-        // 512, 1024, 2048 or 4096 (64 to 512 16-byte vectors per row).
-        g.rowpath = (!momentum && wg_aligned && (m == 512 || m == 1024 || m == 2048 || m == 4096)) ? 1u : 0u;
+        // Whole-row phases A and C: factored matrices of width 512, 1024, 2048
+        // or 4096 (64 to 512 16-byte vectors per row), with or without momentum.
+        g.rowpath = (wg_aligned && (m == 512 || m == 1024 || m == 2048 || m == 4096)) ? 1u : 0u;
         if (g.rowpath) {
-            g.cr = (uint32_t)(kRowChunkBytes / (2 * m));
-            g.rt_rows = g.cr * kRowChunks;
+            g.cr = (uint32_t)((momentum ? kMomGBytes : kRowChunkBytes) / (2 * m));
+            g.rt_rows = g.cr * (momentum ? kMomChunks : kRowChunks);
             g.rtiles = (uint32_t)((n + g.rt_rows - 1) / g.rt_rows);
             g.nfr = 0;
+            // tall matrices: up to 8 threads share a column, each adding every 8th tile
+            uint32_t tpc = 1;
+            while (tpc < 8 && g.rtiles >= 64u * tpc) tpc <<= 1;
+            g.fci = (uint32_t)(kFinChunk / tpc);
+            g.nfc = (uint32_t)((m + g.fci - 1) / g.fci);
         } else {
             g.nfr = (uint32_t)((n + kFinChunk - 1) / kFinChunk);
         }
@@ -152,6 +162,7 @@ struct TensorDev {
     uint32_t cr;        // row path: rows per chunk
     uint32_t rt_rows;   // row path: rows per row tile
     uint32_t rtiles;    // row path: row tiles
+    uint32_t fci;       // row path: columns per finalize item
 };
 
 // Per-tensor scalars of the current step (zeroed at the start of every step).

@@ -311,3 +311,41 @@ def test_fp32_awkward_shapes_and_policies():
         for t in range(1, 4):
             h.step(t, seed=t + policy)
         h.close()
+
+
+def _momentum_row_workload():
+    """Momentum matrices on the whole-row path (the backbone; experts under the momentum
+    variants): every width, ragged tiles and chunks, one-row and tiny matrices, a stack."""
+    B, E = WL.TIER_BACKBONE, WL.TIER_EXPERT
+    specs = [WL.Spec("b300x4096", (300, 4096), B), WL.Spec("b1x4096", (1, 4096), B),
+             WL.Spec("b77x2048", (77, 2048), B), WL.Spec("b1333x1024", (1333, 1024), B),
+             WL.Spec("b2101x512", (2101, 512), B), WL.Spec("s3x130x4096", (3, 130, 4096), B),
+             WL.Spec("e257x4096", (257, 4096), E, expert=0), WL.Spec("v4096", (4096,), B)]
+    return WL.Workload("momrow", specs, WL.HP(policy=WL.POLICY_EXPERT_MOMENTUM), "normal", steps=4)
+
+
+def test_momentum_row_path():
+    """The new M is stored in phase A and sum(U^2) comes from Q_j = sum_i M_ij^2 / R_i."""
+    h = _harness(_momentum_row_workload())
+    assert all(h.opt.info(k).rowpath == 1 and h.opt.info(k).momentum == 1
+               for k, s in enumerate(h.wl.specs) if len(s.shape) >= 2)
+    for t in range(1, 5):
+        h.step(t, seed=7 * t)
+    h.close()
+
+
+def test_momentum_row_path_fallbacks():
+    """eps = 1e-8 (the clamp binds at step 1: phase B runs on the stored new M, not a second
+    update) and a matrix whose gradient is zero at step 1 (R_i == 0 rows: phase B too)."""
+    h = _harness(_momentum_row_workload(), hp_override=dict(eps=1e-8, lr=3e-4, weight_decay=0.05))
+    for t in range(1, 4):
+        h.step(t, seed=3)
+    h.close()
+    h = _harness(_momentum_row_workload())
+    for t in range(1, 4):
+        h.load_grads(t)
+        if t == 1:
+            h.G[0].zero_()
+            h.G[5][1].zero_()
+        h.step(t, seed=9, grads_loaded=True)
+    h.close()
