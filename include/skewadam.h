@@ -260,10 +260,9 @@ const char *skew_kernel_name(int32_t k);
  * workspace; this entry point instead uses a fixed scratch array compiled into
  * the library: SKEW_NOALLOC_SCRATCH_BYTES of device memory on every GPU that
  * loads the library, held until the process exits. That is enough for one
- * tensor of up to about 50,000 x 4,096 with momentum (the paper's 50,304 x
- * 4,096 embedding fits) or about 43,000 x 4,096 without (an expert matrix's
- * whole-row partials take more room); larger tensors are rejected with
- * SKEW_ETOOBIG before any work is enqueued.
+ * 4,096-wide matrix of up to about 65,000 rows (the paper's 50,304 x 4,096
+ * embedding fits; the whole-row partials take 256 bytes per row); larger
+ * tensors are rejected with SKEW_ETOOBIG before any work is enqueued.
  *
  * Arguments: weight / grad as in skew_param_desc_t (device, bf16 or with
  * SKEW_F_FP32 fp32, row-major);

@@ -100,7 +100,7 @@ static void resolve(int ndim, int tier, int policy, uint32_t flags, TPlan &p) {
 }
 
 // Tile geometry (plan_geometry): strip tiles of (tile_rows rows) x (8*LC
-// columns) or flat tiles of 64 Ki elements, and for the row path whole-row tiles.
+// columns) or flat tiles of kFlatTileElems elements, and for the row path whole-row tiles.
 static void geometry(TPlan &p, bool wg_aligned) {
     const TileGeom g = plan_geometry(p.kind, p.momentum, wg_aligned, p.n, p.m, p.numel);
     p.lcl = g.lcl;

@@ -977,16 +977,35 @@ __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem 
         sm.last = (atom_add_acq_rel(&S.cntF, 1u) == T.nfc - 1);
     }
     __syncthreads();
-    if (sm.last && threadIdx.x == 0) {
-        double rs = 0.0, fs = 0.0;
-        float rmn = inf, cmn = inf;
-        for (uint32_t r = 0; r < T.rtiles; ++r) {
-            rs += __ldcg(T.rsum + r);
-            rmn = fminf(rmn, __ldcg(T.rmin + r));
-        }
-        for (uint32_t f = 0; f < T.nfc; ++f) {
-            fs += __ldcg(T.fsum + f);
-            cmn = fminf(cmn, __ldcg(T.fmin + f));
+    if (!sm.last) return;
+    // Last item of the tensor: the whole CTA sums the row tiles' R sums and minima and
+    // the items' sums and minima (thread k takes entries k, k + kThreads, ...; then a
+    // fixed shuffle tree: the same order every step).
+    double rs = 0.0, fs = 0.0;
+    float rmn = inf, cmn = inf;
+    for (uint32_t r = threadIdx.x; r < T.rtiles; r += kThreads) {
+        rs += __ldcg(T.rsum + r);
+        rmn = fminf(rmn, __ldcg(T.rmin + r));
+    }
+    for (uint32_t f = threadIdx.x; f < T.nfc; f += kThreads) {
+        fs += __ldcg(T.fsum + f);
+        cmn = fminf(cmn, __ldcg(T.fmin + f));
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        rmn = fminf(rmn, __shfl_xor_sync(kAll, rmn, o));
+        cmn = fminf(cmn, __shfl_xor_sync(kAll, cmn, o));
+    }
+    if ((threadIdx.x & 31) == 0) {  // colred was last read before the barrier above
+        sm.colred[threadIdx.x >> 5] = rmn;
+        sm.colred[kThreads / 32 + (threadIdx.x >> 5)] = cmn;
+    }
+    rs = block_sum_d(rs, sm.redd);  // its barriers also publish the minima
+    fs = block_sum_d(fs, sm.redd);
+    if (threadIdx.x == 0) {
+        for (int w = 0; w < kThreads / 32; ++w) {
+            rmn = fminf(rmn, sm.colred[w]);
+            cmn = fminf(cmn, sm.colred[kThreads / 32 + w]);
         }
         const double rbar = rs / (double)T.n;
         set_rbar(S, rbar);
@@ -1039,11 +1058,11 @@ __device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm)
     __syncthreads();
     if (threadIdx.x == 0) sm.last = (atom_add_acq_rel(&S.cntF, 1u) == T.nfr + T.nfc - 1);
     __syncthreads();
-    if (sm.last && threadIdx.x == 0) {
-        double s = 0.0;
-        for (uint32_t f = 0; f < T.nfr; ++f) s += __ldcg(T.rsum + f);
-        set_rbar(S, s / (double)T.n);
-    }
+    if (!sm.last) return;
+    double s = 0.0;  // the CTA sums the row items' partials (fixed partition and tree)
+    for (uint32_t f = threadIdx.x; f < T.nfr; f += kThreads) s += __ldcg(T.rsum + f);
+    s = block_sum_d(s, sm.redd);
+    if (threadIdx.x == 0) set_rbar(S, s / (double)T.n);
 }
 
 // ---------------------------------------------------------------------------
@@ -1140,8 +1159,8 @@ __device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
 template <bool VEC>
 __device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t tile, const Pol &pol) {
     Acc2 acc;
-    for (int k = 0; k < kVecPerThread; ++k) {
-        const int64_t e0 = 8 * (int64_t(tile) * kThreads * kVecPerThread + int64_t(k) * kThreads + threadIdx.x);
+    for (int k = 0; k < kFlatVecPerThread; ++k) {
+        const int64_t e0 = 8 * (int64_t(tile) * kThreads * kFlatVecPerThread + int64_t(k) * kThreads + threadIdx.x);
         if (e0 >= T.numel) break;
         const int valid = (int)min(int64_t(8), T.numel - e0);
         float g[8], v[8], y[8];
@@ -1349,8 +1368,8 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
                                 const Pol &pol) {
     const float coefC = __ldcg(&S.coefC);
     const float wdf = T.decay ? A.wdf : 1.0f;
-    for (int k = 0; k < kVecPerThread; ++k) {
-        const int64_t e0 = 8 * (int64_t(tile) * kThreads * kVecPerThread + int64_t(k) * kThreads + threadIdx.x);
+    for (int k = 0; k < kFlatVecPerThread; ++k) {
+        const int64_t e0 = 8 * (int64_t(tile) * kThreads * kFlatVecPerThread + int64_t(k) * kThreads + threadIdx.x);
         if (e0 >= T.numel) break;
         const int valid = (int)min(int64_t(8), T.numel - e0);
         float y[8], v[8], w[8], x[8];

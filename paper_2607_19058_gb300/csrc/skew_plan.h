@@ -12,11 +12,13 @@
 namespace skew {
 
 // Every kernel runs 256-thread CTAs; a thread owns 8 consecutive bf16 elements
-// (one 16-byte vector) of up to kVecPerThread rows (strip tiles) or flat
-// vectors (full-second-moment tiles). A tile is therefore 64 Ki elements.
+// (one 16-byte vector) of up to kVecPerThread rows (strip tiles: 64 Ki elements)
+// or of kFlatVecPerThread flat vectors (full-second-moment tiles: 8 Ki elements,
+// so that the router and the vectors, small, spread over many CTAs).
 constexpr int kThreads = 256;
 constexpr int kVecPerThread = 32;
-constexpr int64_t kFlatTileElems = int64_t(kThreads) * kVecPerThread * 8;
+constexpr int kFlatVecPerThread = 4;
+constexpr int64_t kFlatTileElems = int64_t(kThreads) * kFlatVecPerThread * 8;
 constexpr int kFinChunk = 256;  // rows / columns per finalize item
 
 // Row-tile path (phase A on whole rows, no phase B unless a clamp may bind):
