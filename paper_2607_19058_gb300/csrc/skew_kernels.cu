@@ -594,6 +594,17 @@ __device__ __forceinline__ RowChunk row_chunk(const TensorDev &T, uint32_t tile,
     return RowChunk{i0, left <= 0 ? 0u : (uint32_t)min(left, (int64_t)T.cr)};
 }
 
+// Sum of N values p[0], p[stride], ..., p[(N - 1) stride] (N a power of two) by a
+// balanced tree.
+template <int N>
+__device__ __forceinline__ float tree_sum(const float *p, int stride) {
+    if constexpr (N == 1) {
+        return p[0];
+    } else {
+        return tree_sum<N / 2>(p, stride) + tree_sum<N / 2>(p + (N / 2) * stride, stride);
+    }
+}
+
 // Sum over a warp of K per-lane values, transposed: lane L ends with the total
 // of value j(L) (K = 8: j = 4*b4 + 2*b3 + b2 of L's bits; K = 4: j = 2*b4 + b3;
 // K = 2: j = b4), held by the lanes whose low 2, 3 or 4 bits are zero.
@@ -732,29 +743,27 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         if ((lane & (K == 8 ? 3 : 7)) == 0) sm.part[warp][j] = tot;
         if (__syncthreads_or(!ok)) break;  // every slot before this one has landed
         // slot of chunk c - 1 is free (its pass 2 preceded this barrier): refill it
-        if (tid == 0 && c >= 1 && c - 1 + kRowStages < nch) {
+        // (from warp 1: warp 0 forms the chunk's row scales, which the CTA waits for)
+        if (tid == 32 && c >= 1 && c - 1 + kRowStages < nch) {
             fence_proxy_async_smem();
             row_issue(T, tile, c - 1 + kRowStages, sm, pol);
         }
+        float Rn = 0.f, sum = 0.f;
         if (tid < (int)ch.rows) {  // chunk row r = tid: row-in-pass r % RPP, its k = r / RPP
             const int w0 = (tid % RPP) * WPR, kr = tid / RPP;
-            float sum = 0.f;
-#pragma unroll
-            for (int w = 0; w < WPR; ++w) sum += sm.part[w0 + w][kr];
-            const float mean = sum * inv_m;
-            const float Rn = fmaf(b2, rp, c2 * mean);
-            T.R[ch.i0 + tid] = Rn;
-            rsum += (double)Rn;
-            float inv = 0.f;
-            if (Rn > 0.f && Rn < __int_as_float(0x7F800000)) {
-                rmin = fminf(rmin, Rn);
-                inv = __frcp_rn(Rn);
-            } else if (!(Rn == 0.f && sum == 0.f)) {
-                zero_row = true;  // content in a row with R_i == 0, or a non-finite R_i
-            }
-            sm.inv[tid] = inv;
+            sum = tree_sum<WPR>(&sm.part[w0][kr], 8);
+            Rn = fmaf(b2, rp, c2 * (sum * inv_m));
+            sm.inv[tid] = Rn > 0.f && Rn < __int_as_float(0x7F800000) ? __frcp_rn(Rn) : 0.f;
         }
         __syncthreads();
+        if (tid < (int)ch.rows) {  // the row's R and the tile's statistics, off the barrier's path
+            T.R[ch.i0 + tid] = Rn;
+            rsum += (double)Rn;
+            if (Rn > 0.f && Rn < __int_as_float(0x7F800000))
+                rmin = fminf(rmin, Rn);
+            else if (!(Rn == 0.f && sum == 0.f))
+                zero_row = true;  // content in a row with R_i == 0, or a non-finite R_i
+        }
         // pass 2: P_j += g^2 / R_i, summed in fp32 over four chunks (at most 4 K rows)
         // per column, then folded into (hi, lo)
 #pragma unroll
@@ -1658,28 +1667,26 @@ __device__ void rowsq_mom_tile(const StepArgs &A, const TensorDev &T, TensorScal
         const float tot = warp_sum_transposed<K>(rs, j);
         if ((lane & (K == 4 ? 7 : 15)) == 0) sm.part[warp][j] = tot;
         if (__syncthreads_or(!ok)) break;  // every slot before this one has landed
-        if (tid == 0 && c >= 1 && c - 1 + kMomStages < nch) {
+        // refill from warp 1: warp 0 forms the chunk's row scales, which the CTA waits for
+        if (tid == 32 && c >= 1 && c - 1 + kMomStages < nch) {
             fence_proxy_async_smem();
             mom_issue(T, T.g, tile, c - 1 + kMomStages, sm.buf, sm.full, pol);
         }
+        float Rn = 0.f;
         if (tid < (int)ch.rows) {
             const int w0 = (tid % RPP) * WPR, kr = tid / RPP;
-            float sum = 0.f;
-#pragma unroll
-            for (int w = 0; w < WPR; ++w) sum += sm.part[w0 + w][kr];
-            const float Rn = fmaf(b2, rp, c2 * (sum * inv_m));
-            T.R[ch.i0 + tid] = Rn;
-            rsum += (double)Rn;
-            float inv = 0.f;
-            if (Rn > 0.f && Rn < __int_as_float(0x7F800000)) {
-                rmin = fminf(rmin, Rn);
-                inv = __frcp_rn(Rn);
-            } else {
-                zero_row = true;  // R_i == 0 or not finite: its momentum may still be nonzero
-            }
-            sm.inv[tid] = inv;
+            Rn = fmaf(b2, rp, c2 * (tree_sum<WPR>(&sm.part[w0][kr], 8) * inv_m));
+            sm.inv[tid] = Rn > 0.f && Rn < __int_as_float(0x7F800000) ? __frcp_rn(Rn) : 0.f;
         }
         __syncthreads();
+        if (tid < (int)ch.rows) {  // the row's R and the tile's statistics, off the barrier's path
+            T.R[ch.i0 + tid] = Rn;
+            rsum += (double)Rn;
+            if (Rn > 0.f && Rn < __int_as_float(0x7F800000))
+                rmin = fminf(rmin, Rn);
+            else
+                zero_row = true;  // R_i == 0 or not finite: its momentum may still be nonzero
+        }
         // pass 2: M <- b1 M + (1 - b1) g (stored), Q_j += M^2 / R_i
 #pragma unroll
         for (int k = 0; k < K; ++k) {
