@@ -6,7 +6,7 @@ momentum, exact router / vector second moments, update-RMS clipping, decoupled
 weight decay, dithered bf16 write-back) over a synthetic parameter set shaped
 like the paper's 6.78B-parameter MoE (App. B shapes: 6,784,327,680 bf16
 parameters in 408 tensors). Weights ~ N(0, 0.02^2), gradients ~ N(0, 1e-3^2),
-resident in HBM; 27.1 GB of weights + gradients per step is far larger than the
+resident in HBM; 27.1 GB of weights + gradients per step (App. B shapes) is far larger than the
 129 MiB L2, so no flush is needed between steps.
 
 Reported (one JSON line, rank 0):
@@ -119,6 +119,13 @@ def clocks_stop(handle):
 # ---------------------------------------------------------------------------
 # byte accounting
 # ---------------------------------------------------------------------------
+def policy_name(wl):
+    from paper_2607_19058_gb300 import workloads as WL
+    return {WL.POLICY_TIERED: "tiered", WL.POLICY_EXPERT_MOMENTUM: "expert_momentum",
+            WL.POLICY_FACTORED_ROUTER: "factored_router", WL.POLICY_UNIFORM: "uniform",
+            WL.POLICY_ADAFACTOR: "adafactor"}[wl.hp.policy]
+
+
 def byte_model(opt, n_tensors):
     """Algorithmic minimum bytes of one step and of each kernel's own traffic."""
     N = N_mom = N_full = N_fact = N_nomom = N_row = N_rowm = 0
@@ -268,7 +275,7 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_full, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "params": wl.numel, "tensors": len(wl.specs), "policy": "tiered"},
+        "config": {"workload": wl.name, "params": wl.numel, "tensors": len(wl.specs), "policy": policy_name(wl)},
         "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc},
         "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "note": "CPU oracle (plain fp64 C, single thread) on bounded samples of the workload; ms_per_step is the "
@@ -341,6 +348,7 @@ def run_ours(args):
     params = [(W[k], G[k], s.tier, S.F_NO_DECAY if s.no_decay else 0) for k, s in enumerate(wl.specs)]
     opt = S.SkewAdam(params, S.hparams(hp.beta1, hp.beta2, hp.eps, hp.clip_d, hp.weight_decay, hp.policy))
     bm = byte_model(opt, len(wl.specs))
+    wg_bytes = sum(w.numel() * w.element_size() + g.numel() * g.element_size() for w, g in zip(W, G))
     stream = torch.cuda.current_stream()
     torch.cuda.synchronize()
 
@@ -455,9 +463,9 @@ def run_ours(args):
             "value": job_rate(world, bm["N"], ms), "unit": "params/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": wl.name, "params": bm["N"], "tensors": len(wl.specs), "policy": "tiered",
+            "config": {"workload": wl.name, "params": bm["N"], "tensors": len(wl.specs), "policy": policy_name(wl),
                        "state_bytes": opt.state_bytes, "workspace_bytes": opt.workspace_bytes,
-                       "l2": "inputs larger than L2 (27.1 GB of bf16 weights + grads vs 129 MiB), no flush",
+                       "l2": f"inputs larger than L2 ({wg_bytes / 1e9:.1f} GB of weights + grads vs 129 MiB), no flush",
                        "weights_grads": "bf16, W~N(0,0.02^2), G~N(0,1e-3^2)"},
             "hbm": {"min_bytes_per_step": bm["step_min"], "achieved_gbs": step_gbs,
                     "frac_of_8tbs": step_gbs / NOMINAL_HBM_GBS, "frac_of_measured": step_gbs / peak,
