@@ -52,6 +52,7 @@ def parse():
     p.add_argument("--workload", default="appb", help="shape set (appb = the paper's 6.78B App. B shapes)")
     p.add_argument("--seed", type=int, default=20260207)
     p.add_argument("--e2e-steps", type=int, default=6)
+    p.add_argument("--e2e-groups", type=int, default=4, help="tensor groups of the end-to-end leg's pipeline")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="target oracle time of the CPU baseline sample")
@@ -312,7 +313,7 @@ def job_rate(world, params_per_rank, ms):
 def flat_views(wl, dev):
     """One device buffer holding every tensor of the workload (bf16, or fp32 for an fp32
     tensor) at 512-byte aligned offsets (as the allocator places separate tensors);
-    returns it and the per-tensor views."""
+    returns it, the per-tensor views and their byte offsets (with the total last)."""
     import torch
     offs, total = [], 0
     for s in wl.specs:
@@ -321,7 +322,21 @@ def flat_views(wl, dev):
         total += s.numel * (4 if s.fp32 else 2)
     buf = torch.empty(max(total, 1), dtype=torch.uint8, device=dev)
     views = [buf[o:o + s.numel * (4 if s.fp32 else 2)].view(s.dtype).view(s.shape) for o, s in zip(offs, wl.specs)]
-    return buf, views
+    return buf, views, offs + [total]
+
+
+def e2e_groups(offs, n_groups):
+    """Splits the tensors (byte offsets `offs`, total last) into at most n_groups runs of
+    consecutive tensors of about equal bytes: [(first, end), ...]."""
+    total, n = offs[-1], len(offs) - 1
+    bounds, k = [0], 0
+    for gi in range(1, n_groups):
+        while k < n and offs[k] < total * gi / n_groups:
+            k += 1
+        if bounds[-1] < k < n:
+            bounds.append(k)
+    bounds.append(n)
+    return list(zip(bounds[:-1], bounds[1:]))
 
 
 def run_ours(args):
@@ -386,24 +401,29 @@ def run_ours(args):
     step_gbs = bm["step_min"] / (ms * 1e-3) / 1e9
 
     # end to end through the C ABI with host buffers: every step copies all gradients in
-    # from pinned host memory (one copy) and all updated weights back out (one copy); the
-    # copy-in of step t+1 runs on its own stream beside the copy-out of step t (each waits
-    # only for the step that frees its buffer). For one copy per direction this leg keeps
-    # every weight (gradient) as a 512-byte aligned view of one device buffer, in a handle
-    # of its own over the same parameters.
+    # from pinned host memory and all updated weights back out. The step has no coupling
+    # across tensors, so this leg runs it as --e2e-groups handles over runs of consecutive
+    # tensors, each a 512-byte aligned slice of one device buffer per kind: group g's
+    # gradients come in (one copy), its step runs, its weights go out (one copy), while the
+    # next group's gradients are already coming in. Each copy waits only for the step that
+    # frees its buffer, so the host link stays busy in both directions.
     e2e = None
     if not args.no_e2e and args.e2e_steps > 0:
-        Wbuf, Wf = flat_views(wl, dev)
-        Gbuf, Gf = flat_views(wl, dev)
+        Wbuf, Wf, offs = flat_views(wl, dev)
+        Gbuf, Gf, _ = flat_views(wl, dev)
         for k in range(len(wl.specs)):
             Wf[k].copy_(W[k])
             Gf[k].copy_(G[k])
-        opt_e2e = S.SkewAdam([(Wf[k], Gf[k], s.tier, S.F_NO_DECAY if s.no_decay else 0)
-                              for k, s in enumerate(wl.specs)],
-                             S.hparams(hp.beta1, hp.beta2, hp.eps, hp.clip_d, hp.weight_decay, hp.policy))
+        groups = e2e_groups(offs, max(1, args.e2e_groups))
+        opts = [S.SkewAdam([(Wf[k], Gf[k], wl.specs[k].tier, S.F_NO_DECAY if wl.specs[k].no_decay else 0)
+                            for k in range(k0, k1)],
+                           S.hparams(hp.beta1, hp.beta2, hp.eps, hp.clip_d, hp.weight_decay, hp.policy))
+                for k0, k1 in groups]
+        spans = [(offs[k0], offs[k1] if k1 < len(wl.specs) else offs[-1]) for k0, k1 in groups]
         for _ in range(args.warmup):
             step += 1
-            opt_e2e.step(step, hp.lr, args.seed)
+            for o in opts:
+                o.step(step, hp.lr, args.seed)
         hg = torch.empty(Gbuf.numel(), dtype=torch.uint8, pin_memory=True)
         hw = torch.empty(Wbuf.numel(), dtype=torch.uint8, pin_memory=True)
         hg.copy_(Gbuf)
@@ -414,36 +434,41 @@ def run_ours(args):
         ev = lambda: torch.cuda.Event(enable_timing=False)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(s_in)
-        stepped = drained = None
+        stepped = [None] * len(groups)
+        drained = [None] * len(groups)
         for _ in range(args.e2e_steps):
             step += 1
-            if stepped is not None:
-                s_in.wait_event(stepped)       # the previous step has read its gradients
-            with torch.cuda.stream(s_in):
-                Gbuf.copy_(hg, non_blocking=True)
-            loaded = ev()
-            loaded.record(s_in)
-            stream.wait_event(loaded)
-            if drained is not None:
-                stream.wait_event(drained)     # the previous weights are back on the host
-            opt_e2e.step(step, hp.lr, args.seed)
-            stepped = ev()
-            stepped.record(stream)
-            s_out.wait_event(stepped)
-            with torch.cuda.stream(s_out):
-                hw.copy_(Wbuf, non_blocking=True)
-            drained = ev()
-            drained.record(s_out)
+            for gi, (lo, hi) in enumerate(spans):
+                if stepped[gi] is not None:
+                    s_in.wait_event(stepped[gi])       # the group's last step has read its gradients
+                with torch.cuda.stream(s_in):
+                    Gbuf[lo:hi].copy_(hg[lo:hi], non_blocking=True)
+                loaded = ev()
+                loaded.record(s_in)
+                stream.wait_event(loaded)
+                if drained[gi] is not None:
+                    stream.wait_event(drained[gi])     # the group's last weights are back on the host
+                opts[gi].step(step, hp.lr, args.seed)
+                stepped[gi] = ev()
+                stepped[gi].record(stream)
+                s_out.wait_event(stepped[gi])
+                with torch.cuda.stream(s_out):
+                    hw[lo:hi].copy_(Wbuf[lo:hi], non_blocking=True)
+                drained[gi] = ev()
+                drained[gi].record(s_out)
         b.record(s_out)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(a.elapsed_time(b) / args.e2e_steps, world, dev)
         e2e = {"value": job_rate(world, bm["N"], e2e_ms), "unit": "params/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int(Gbuf.numel()), "d2h_bytes_per_step": int(Wbuf.numel()),
-               "path": "skew_step via ctypes; every step copies all gradients in from pinned host memory and all "
-                       "updated weights back to pinned host memory, one copy per direction, the copy-in of the "
-                       "next step beside the copy-out of the last"}
-        opt_e2e.sync_status()
-        opt_e2e.close()
+               "groups": len(groups),
+               "path": f"skew_step via ctypes on {len(groups)} handles over runs of consecutive tensors; every "
+                       "step copies all gradients in from pinned host memory and all updated weights back to "
+                       "pinned host memory, one copy per direction per group, a group's copies beside the "
+                       "other groups' steps"}
+        for o in opts:
+            o.sync_status()
+            o.close()
         del hg, hw, Wf, Gf, Wbuf, Gbuf
 
     cpu = None
