@@ -213,6 +213,21 @@ def oracle_sample_specs(wl, target_params):
     return chosen, tot
 
 
+def host_info():
+    """The host the CPU oracle runs on: its logical CPU count and CPU model."""
+    import platform
+    model = None
+    try:
+        for ln in open("/proc/cpuinfo"):
+            key = ln.split(":")[0].strip().lower()
+            if key in ("model name", "cpu model", "hardware"):
+                model = ln.split(":", 1)[1].strip()
+                break
+    except OSError:
+        pass
+    return {"nproc": os.cpu_count(), "cpu": model or platform.machine()}
+
+
 def time_oracle(wl, tids, inputs, step, lr, seed):
     import oracle as O
     from paper_2607_19058_gb300 import workloads as WL
@@ -277,7 +292,8 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_full, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": wl.name, "params": wl.numel, "tensors": len(wl.specs), "policy": policy_name(wl)},
-        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc},
+        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc,
+                         "host": host_info()},
         "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "note": "CPU oracle (plain fp64 C, single thread) on bounded samples of the workload; ms_per_step is the "
                 "full-workload equivalent at the sampled rate",
@@ -392,8 +408,11 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
 
-    # per-kernel live durations
+    # per-kernel live durations; per-step spans (first launch to last, from the same events)
     kmean = {n: statistics.fmean(r[i] for r in rows) for i, n in enumerate(names)}
+    spans = [sum(r) for r in rows]
+    step_stats = {"median_ms": statistics.median(spans), "mean_ms": statistics.fmean(spans),
+                  "min_ms": min(spans), "max_ms": max(spans)} if spans else None
     dom = max(kmean, key=kmean.get)
     peak, peak_src = peaks()
     dom_bytes = bm["kernels"][dom]
@@ -478,7 +497,7 @@ def run_ours(args):
         src = {k: (W[k], G[k]) for k in tids}
         inputs = cpu_inputs(wl, tids, src=src)
         secs = time_oracle(wl, tids, inputs, 1, hp.lr, args.seed)
-        cpu = {"value": tot / secs, "unit": "params/s", "cores": 1, "kind": "oracle",
+        cpu = {"value": tot / secs, "unit": "params/s", "cores": 1, "kind": "oracle", "host": host_info(),
                "sample": f"one step of {len(tids)} of the {len(wl.specs)} tensors ({tot} params, tier mix kept) "
                          f"in {secs:.1f} s, single-threaded fp64 C"}
 
@@ -499,6 +518,7 @@ def run_ours(args):
                          "frac": achieved / peak, "traffic": recorded_traffic(dom, args.workload), "algorithmic_bytes_per_launch": dom_bytes,
                          "launch_ms": kmean[dom], "peak_source": peak_src},
             "kernels_ms": kmean,
+            "step_spans": step_stats,
             "e2e": e2e,
             "cpu_baseline": cpu,
             "gpu_launches": args.steps * S.skew_launches_per_step(opt.h),
