@@ -219,6 +219,18 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
 int skew_sync_status(skew_handle_t *h, void *stream);
 
 /*
+ * Self-test of the failure path of the bounded device waits: enqueues on
+ * `stream` one thread that waits, exactly as the whole-row kernels wait for a
+ * copied chunk, on an mbarrier phase that nothing completes. The wait gives up
+ * after its poll limit (about two seconds at most) and records the timeout in
+ * the handle's status word, so the next skew_sync_status returns SKEW_ETIMEOUT
+ * and clears it; the context stays usable and later steps are unaffected.
+ * Asynchronous. Errors: SKEW_EINVAL (null), SKEW_ESTATE (not bound),
+ * SKEW_ECUDA (launch failure).
+ */
+int skew_selftest_wait_timeout(skew_handle_t *h, void *stream);
+
+/*
  * Per-tensor scalars of the last completed step, for inspection and tests:
  * out[0] = mean(R) (factored tensors, else 0), out[1] = sum of U^2 over the
  * tensor, out[2] = RMS(U), out[3] = clip factor 1/max(1, RMS/d). Synchronises

@@ -530,6 +530,14 @@ int skew_sync_status(skew_handle_t *h, void *stream) {
     return SKEW_OK;
 }
 
+int skew_selftest_wait_timeout(skew_handle_t *h, void *stream) {
+    if (!h) return SKEW_EINVAL;
+    if (!h->bound) return fail(h, SKEW_ESTATE, "not bound");
+    const cudaError_t e = (cudaError_t)launch_wait_selftest(reinterpret_cast<uint32_t *>(h->ws + h->ws_err), stream);
+    if (e != cudaSuccess) return cuda_fail(h, e, "kernel launch");
+    return SKEW_OK;
+}
+
 int skew_tensor_scalars(skew_handle_t *h, int32_t tid, double out[4], void *stream) {
     return skew_matrix_scalars(h, tid, 0, out, stream);
 }

@@ -2068,7 +2068,24 @@ __global__ void __launch_bounds__(kThreads, SKEW_MINB_APPLY)
     }
 }
 
+// Self-test of the bounded wait: one thread waits, exactly as the row kernels wait for
+// a chunk, on an mbarrier phase that nothing completes (no arrival, no transaction);
+// the wait gives up after kMbarPolls polls and the timeout lands in the status word.
+__global__ void k_wait_selftest(uint32_t *err) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_mbar_init();
+        if (!mbar_wait(&bar, 0u)) atomicOr(err, 2u);
+    }
+}
+
 }  // namespace
+
+int launch_wait_selftest(uint32_t *err, void *stream) {
+    k_wait_selftest<<<1, 32, 0, (cudaStream_t)stream>>>(err);
+    return (int)cudaGetLastError();
+}
 
 int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *const *ev) {
     cudaStream_t s = (cudaStream_t)stream;

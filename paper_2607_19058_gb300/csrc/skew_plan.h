@@ -223,4 +223,8 @@ constexpr int kLaunches = 7;
 // and after each of the seven. Returns a cudaError_t value.
 int launch_phases(const StepArgs &A, const LaunchPlan &L, void *stream, void *const *ev);
 
+// Enqueues the bounded-wait self-test (one thread waits on an mbarrier phase that
+// never completes and records the timeout in *err). Returns a cudaError_t value.
+int launch_wait_selftest(uint32_t *err, void *stream);
+
 }  // namespace skew

@@ -29,7 +29,7 @@ KIND_FULL, KIND_FACTORED = 0, 1
 EXPORTS = ["skew_create", "skew_destroy", "skew_state_bytes", "skew_workspace_bytes", "skew_bind", "skew_step",
            "skew_sync_status", "skew_tensor_scalars", "skew_matrix_scalars", "skew_tensor_info", "skew_num_tensors", "skew_last_error",
            "skew_profile_begin", "skew_profile_end", "skew_kernel_name", "skew_step_tensor_noalloc",
-           "skew_launches_per_step"]
+           "skew_launches_per_step", "skew_selftest_wait_timeout"]
 
 
 class SkewError(RuntimeError):
@@ -85,6 +85,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
         L.skew_step.restype = C.c_int
         L.skew_sync_status.argtypes = [vp, vp]
         L.skew_sync_status.restype = C.c_int
+        L.skew_selftest_wait_timeout.argtypes = [vp, vp]
+        L.skew_selftest_wait_timeout.restype = C.c_int
         L.skew_tensor_scalars.argtypes = [vp, i32, C.POINTER(C.c_double), vp]
         L.skew_tensor_scalars.restype = C.c_int
         L.skew_matrix_scalars.argtypes = [vp, i32, i32, C.POINTER(C.c_double), vp]
@@ -149,6 +151,10 @@ def skew_step(h, step: int, lr: float, seed: int, stream: int) -> None:
 
 def skew_sync_status(h, stream: int) -> None:
     _check(load().skew_sync_status(h, stream), h)
+
+
+def skew_selftest_wait_timeout(h, stream: int) -> None:
+    _check(load().skew_selftest_wait_timeout(h, stream), h)
 
 
 def skew_tensor_scalars(h, tid: int, stream: int):

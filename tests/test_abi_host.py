@@ -195,6 +195,9 @@ def test_step_before_bind_and_bad_bind_sizes():
     with pytest.raises(S.SkewError) as e:
         S.skew_step(h, 1, 1e-3, 0, 0)
     assert e.value.code == S.SKEW_ESTATE
+    with pytest.raises(S.SkewError) as e:   # the wait self-test too needs a bound handle
+        S.skew_selftest_wait_timeout(h, 0)
+    assert e.value.code == S.SKEW_ESTATE
     with pytest.raises(S.SkewError) as e:   # wrong sizes are rejected before any CUDA call
         S.skew_bind(h, 0x100000, S.skew_state_bytes(h) + 4, 0x200000, S.skew_workspace_bytes(h), 0)
     assert e.value.code == S.SKEW_EINVAL
