@@ -75,3 +75,27 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
         workload, steps, warmup, seed, gpus, ref_seconds = "toy", 1, 0, 0, 2, 1.0
     b.run_reference(Args())                                 # returns before any work or output
     assert capsys.readouterr().out == ""
+
+
+@pytest.mark.parametrize("n_groups", [1, 2, 4, 8, 1000])
+def test_e2e_groups_partition(n_groups):
+    """The end-to-end leg's tensor groups: consecutive runs covering every tensor once,
+    at most n_groups of them, of about equal bytes on the App. B shapes."""
+    b = _bench()
+    from paper_2607_19058_gb300 import workloads as WL
+    for wl in (WL.appb(), WL.toy()):
+        offs, total = [], 0
+        for s in wl.specs:
+            total = (total + 511) // 512 * 512
+            offs.append(total)
+            total += s.numel * (4 if s.fp32 else 2)
+        offs.append(total)
+        groups = b.e2e_groups(offs, n_groups)
+        n = len(wl.specs)
+        assert 1 <= len(groups) <= min(n_groups, n)
+        assert groups[0][0] == 0 and groups[-1][1] == n
+        assert all(k1 == k0n for (_, k1), (k0n, _) in zip(groups, groups[1:]))
+        assert all(k0 < k1 for k0, k1 in groups)
+        if wl.name == "appb" and n_groups <= 8:
+            sizes = [(offs[k1] if k1 < n else offs[-1]) - offs[k0] for k0, k1 in groups]
+            assert max(sizes) <= 1.1 * total / len(groups)
