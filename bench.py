@@ -213,6 +213,17 @@ def oracle_sample_specs(wl, target_params):
     return chosen, tot
 
 
+def mem_available():
+    """MemAvailable of this host in bytes (None where /proc/meminfo is missing)."""
+    try:
+        for ln in open("/proc/meminfo"):
+            if ln.startswith("MemAvailable:"):
+                return int(ln.split()[1]) * 1024
+    except OSError:
+        pass
+    return None
+
+
 def host_info():
     """The host the CPU oracle runs on: its logical CPU count and CPU model."""
     import platform
@@ -428,7 +439,14 @@ def run_ours(args):
     # next group's gradients are already coming in. Each copy waits only for the step that
     # frees its buffer, so the host link stays busy in both directions.
     e2e = None
-    if not args.no_e2e and args.e2e_steps > 0:
+    # pinned host memory of this leg: gradients in and weights out, for every rank on this host
+    host_need = wg_bytes * int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+    host_avail = mem_available()
+    if not args.no_e2e and args.e2e_steps > 0 and host_avail is not None and host_need > 0.8 * host_avail:
+        e2e = {"value": None, "unit": "params/s",
+               "skipped": f"host memory: {host_need / 1e9:.0f} GB of pinned buffers for the ranks on this host, "
+                          f"{host_avail / 1e9:.0f} GB available"}
+    elif not args.no_e2e and args.e2e_steps > 0:
         Wbuf, Wf, offs = flat_views(wl, dev)
         Gbuf, Gf, _ = flat_views(wl, dev)
         for k in range(len(wl.specs)):
