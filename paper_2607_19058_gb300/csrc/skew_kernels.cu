@@ -709,13 +709,19 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
     float rmin = __int_as_float(0x7F800000);  // threads < CS: smallest positive R of it
     bool zero_row = false;
 
+    // the tile's rows and R, held in registers (the stores to R in the loop could
+    // otherwise make the compiler reload them from the descriptor every chunk)
+    const int64_t row0 = int64_t(tile) * T.rt_rows, n = T.n;
+    const uint32_t cr = T.cr;
+    float *__restrict__ Rg = T.R;
     uint32_t c = 0;
     for (; c < nch; ++c) {
         const int st = c % kRowStages;
         const uint32_t par = (c / kRowStages) & 1u;
-        const RowChunk ch = row_chunk(T, tile, c);
+        const int64_t ci0 = row0 + int64_t(c) * cr;
+        const RowChunk ch{ci0, (uint32_t)min(n - ci0, (int64_t)cr)};
         float rp = 0.f;
-        if (tid < (int)ch.rows) rp = __ldcg(T.R + ch.i0 + tid);
+        if (tid < (int)ch.rows) rp = __ldcg(Rg + ch.i0 + tid);
         const bool ok = mbar_wait(&sm.full[st], par);
         const uint4 *buf = sm.buf[st];
         // pass 1: row sums and column sums of g^2 (rows lay.rp + RPP k of the chunk)
@@ -757,7 +763,7 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         }
         __syncthreads();
         if (tid < (int)ch.rows) {  // the row's R and the tile's statistics, off the barrier's path
-            T.R[ch.i0 + tid] = Rn;
+            Rg[ch.i0 + tid] = Rn;
             rsum += (double)Rn;
             if (Rn > 0.f && Rn < __int_as_float(0x7F800000))
                 rmin = fminf(rmin, Rn);
