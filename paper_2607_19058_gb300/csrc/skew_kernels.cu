@@ -25,6 +25,7 @@
 // with L2-only (.cg) loads. When no element of a tile can reach the 1/sqrt(eps)
 // clamp (all but degenerate tiles), phase C takes a clamp-free path.
 #include <cuda_runtime.h>
+#include <type_traits>
 #include <stdint.h>
 
 #include "skew_plan.h"
@@ -724,26 +725,34 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         if (tid < (int)ch.rows) rp = __ldcg(Rg + ch.i0 + tid);
         const bool ok = mbar_wait(&sm.full[st], par);
         const uint4 *buf = sm.buf[st];
+        // a full chunk (every chunk but a tensor's last) needs no row bound checks
+        const bool full = ch.rows == (uint32_t)CS;
         // pass 1: row sums and column sums of g^2 (rows lay.rp + RPP k of the chunk)
         float rs[K];
+        auto pass1 = [&](auto full_c) {
 #pragma unroll
-        for (int k = 0; k < K; ++k) {
-            const int r = lay.rp + RPP * k;
-            float2 r2 = make_float2(0.f, 0.f);
-            if (r < (int)ch.rows) {
+            for (int k = 0; k < K; ++k) {
+                const int r = lay.rp + RPP * k;
+                float2 r2 = make_float2(0.f, 0.f);
+                if (decltype(full_c)::value || r < (int)ch.rows) {
 #pragma unroll
-                for (int v = 0; v < NV; ++v) {
-                    float2 g[4];
-                    unpack_bf8x2(buf[r * V + v * TPB + lay.vi], g);
+                    for (int v = 0; v < NV; ++v) {
+                        float2 g[4];
+                        unpack_bf8x2(buf[r * V + v * TPB + lay.vi], g);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {  // g^2 into the column and row sums, one rounding each
-                        cs[v][q] = __ffma2_rn(g[q], g[q], cs[v][q]);
-                        r2 = __ffma2_rn(g[q], g[q], r2);
+                        for (int q = 0; q < 4; ++q) {  // g^2 into the column and row sums, one rounding each
+                            cs[v][q] = __ffma2_rn(g[q], g[q], cs[v][q]);
+                            r2 = __ffma2_rn(g[q], g[q], r2);
+                        }
                     }
                 }
+                rs[k] = r2.x + r2.y;
             }
-            rs[k] = r2.x + r2.y;
-        }
+        };
+        if (full)
+            pass1(std::true_type{});
+        else
+            pass1(std::false_type{});
         int j;
         const float tot = warp_sum_transposed<K>(rs, j);
         if ((lane & (K == 8 ? 3 : 7)) == 0) sm.part[warp][j] = tot;
@@ -772,21 +781,27 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         }
         // pass 2: P_j += g^2 / R_i, summed in fp32 over four chunks (at most 4 K rows)
         // per column, then folded into (hi, lo)
+        auto pass2 = [&](auto full_c) {
 #pragma unroll
-        for (int k = 0; k < K; ++k) {
-            const int r = lay.rp + RPP * k;
-            if (r < (int)ch.rows) {
-                const float iv = sm.inv[r];
-                const float2 iv2 = make_float2(iv, iv);
+            for (int k = 0; k < K; ++k) {
+                const int r = lay.rp + RPP * k;
+                if (decltype(full_c)::value || r < (int)ch.rows) {
+                    const float iv = sm.inv[r];
+                    const float2 iv2 = make_float2(iv, iv);
 #pragma unroll
-                for (int v = 0; v < NV; ++v) {
-                    float2 g[4];
-                    unpack_bf8x2(buf[r * V + v * TPB + lay.vi], g);
+                    for (int v = 0; v < NV; ++v) {
+                        float2 g[4];
+                        unpack_bf8x2(buf[r * V + v * TPB + lay.vi], g);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) t[v][q] = __ffma2_rn(__fmul2_rn(g[q], g[q]), iv2, t[v][q]);
+                        for (int q = 0; q < 4; ++q) t[v][q] = __ffma2_rn(__fmul2_rn(g[q], g[q]), iv2, t[v][q]);
+                    }
                 }
             }
-        }
+        };
+        if (full)
+            pass2(std::true_type{});
+        else
+            pass2(std::false_type{});
         if ((c & 3u) == 3u || c + 1 == nch) {
 #pragma unroll
             for (int v = 0; v < NV; ++v)
