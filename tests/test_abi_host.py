@@ -236,3 +236,43 @@ def test_fp32_tensors_plan():
     with pytest.raises(S.SkewError) as e:
         S.skew_create([_one((8, 8), weight=0x1002, flags=S.F_FP32)], S.hparams())
     assert e.value.code == S.SKEW_EINVAL and "4-byte" in str(e.value)
+
+
+def _noalloc(**kw):
+    """skew_step_tensor_noalloc with fake device pointers: every check below happens on the
+    host before any CUDA call; returns the error code (SKEW_OK never: no GPU here)."""
+    a = dict(weight=0x100000, grad=0x200000, ndim=2, rows=64, cols=128, tier=S.TIER_EXPERT, flags=0,
+             hp=S.hparams(), state=0x300000, tensor_id=0, step=1, lr=1e-3, seed=0, stream=0)
+    a.update(kw)
+    if "state_bytes" not in a:   # the closed form for an expert matrix under the tiered policy: R and C
+        a["state_bytes"] = 4 * (a["rows"] + (a["cols"] if a["ndim"] == 2 else 0))
+    try:
+        S.skew_step_tensor_noalloc(a["weight"], a["grad"], a["ndim"], a["rows"], a["cols"], a["tier"], a["flags"],
+                                   a["hp"], a["state"], a["state_bytes"], a["tensor_id"], a["step"], a["lr"],
+                                   a["seed"], a["stream"])
+    except S.SkewError as e:
+        return e.code
+    return S.SKEW_OK
+
+
+@pytest.mark.parametrize("kw", [dict(weight=0), dict(grad=0), dict(state=0), dict(weight=0x100001),
+                                dict(state=0x300002), dict(ndim=3), dict(ndim=0), dict(tier=3), dict(flags=4),
+                                dict(step=0), dict(lr=-1.0), dict(lr=float("nan")), dict(rows=0),
+                                dict(hp=S.hparams(beta2=1.0)), dict(hp=S.hparams(policy=5)),
+                                dict(state_bytes=4 * (64 + 128) + 4)])
+def test_noalloc_rejects_bad_arguments_on_the_host(kw):
+    assert _noalloc(**kw) == S.SKEW_EINVAL
+
+
+def test_noalloc_scratch_limit_on_the_host():
+    """The fixed scratch holds a 4096-wide matrix of about 65,000 rows (the paper's 50,304 x 4096
+    embedding included): smaller ones pass every host check (and then need a GPU: SKEW_ECUDA
+    here), larger ones are SKEW_ETOOBIG before any CUDA call."""
+    import torch
+    mom = S.TIER_BACKBONE  # momentum + factored: state M, R, C
+    if not torch.cuda.is_available():  # (with a GPU the fake pointers would reach the kernels)
+        fits = _noalloc(rows=50304, cols=4096, tier=mom, state_bytes=4 * (50304 * 4096 + 50304 + 4096))
+        assert fits == S.SKEW_ECUDA
+    big = _noalloc(rows=80000, cols=4096, tier=mom, state_bytes=4 * (80000 * 4096 + 80000 + 4096))
+    assert big == S.SKEW_ETOOBIG
+    assert _noalloc(rows=1 << 20, cols=8192) == S.SKEW_ETOOBIG
