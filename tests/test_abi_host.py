@@ -276,3 +276,60 @@ def test_noalloc_scratch_limit_on_the_host():
     big = _noalloc(rows=80000, cols=4096, tier=mom, state_bytes=4 * (80000 * 4096 + 80000 + 4096))
     assert big == S.SKEW_ETOOBIG
     assert _noalloc(rows=1 << 20, cols=8192) == S.SKEW_ETOOBIG
+
+
+def test_random_plans_tile_the_state():
+    """Random parameter lists (vectors, matrices, stacks; every tier; no-decay and fp32
+    flags; every policy): the planner's state is the oracle's closed form, each tensor's
+    kind / momentum / decay is the oracle's, and its arrays tile the state buffer exactly.
+    The row path is chosen exactly for bf16 factored matrices 512 to 4096 wide (powers of
+    two) with 16-byte aligned pointers."""
+    hyp = pytest.importorskip("hypothesis")
+    st = hyp.strategies
+
+    tensor = st.tuples(st.sampled_from([1, 2, 3]), st.integers(1, 3000), st.sampled_from([1, 7, 64, 512, 1000, 1024,
+                                                                                            2048, 4096, 5000]),
+                       st.integers(1, 3), st.sampled_from([S.TIER_BACKBONE, S.TIER_EXPERT, S.TIER_ROUTER]),
+                       st.booleans(), st.booleans(), st.booleans())
+
+    @hyp.settings(max_examples=150, deadline=None, derandomize=True)
+    @hyp.given(st.lists(tensor, max_size=10), st.sampled_from([S.POLICY_TIERED, S.POLICY_EXPERT_MOMENTUM,
+                                                              S.POLICY_FACTORED_ROUTER, S.POLICY_UNIFORM,
+                                                              S.POLICY_ADAFACTOR]))
+    def check(tensors, policy):
+        descs, specs, meta = [], [], []
+        for k, (nd, n, m, e, tier, nodecay, fp32, misalign) in enumerate(tensors):
+            base = 0x10000000 * (k + 1)
+            w, g = base + (4 if misalign else 0), base + 0x8000000
+            flags = (S.F_NO_DECAY if nodecay else 0) | (S.F_FP32 if fp32 else 0)
+            shp = (n, m) if nd >= 2 else (n, 0)
+            descs.append(S.ParamDesc(w, g, (C.c_int64 * 2)(*shp), nd, tier, flags, e if nd == 3 else 0))
+            mats = [((n, m) if nd >= 2 else (n,), tier)] * (e if nd == 3 else 1)
+            specs += mats
+            meta.append((nd, n, m if nd >= 2 else 1, e if nd == 3 else 1, tier, nodecay, fp32, misalign))
+        h = S.skew_create(descs, S.hparams(policy=policy))
+        try:
+            assert S.skew_state_bytes(h) == O.state_bytes(specs, policy)
+            total = S.skew_state_bytes(h) // 4
+            spans = []
+            for k, (nd, n, m, E, tier, nodecay, fp32, misalign) in enumerate(meta):
+                i = S.skew_tensor_info(h, k)
+                kind, mo, dec = O.resolve(2 if nd == 3 else nd, tier, policy, nodecay)
+                assert (i.kind, i.momentum, i.decay) == (kind, mo, dec)
+                assert i.numel == E * n * m and (i.rows, i.cols) == (n, m)
+                want_row = kind == O.KIND_FACTORED and not fp32 and not misalign and m in (512, 1024, 2048, 4096)
+                assert bool(i.rowpath) == want_row
+                for off, cnt in ((i.m_offset, i.numel), (i.v_offset, i.numel), (i.r_offset, E * n),
+                                 (i.c_offset, E * m)):
+                    if off >= 0:
+                        spans.append((off, off + cnt))
+            spans.sort()
+            if spans:
+                assert spans[0][0] == 0 and spans[-1][1] == total
+                assert all(a[1] == b[0] for a, b in zip(spans, spans[1:]))
+            else:
+                assert total == 0
+        finally:
+            S.skew_destroy(h)
+
+    check()
