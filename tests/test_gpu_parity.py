@@ -218,6 +218,20 @@ def test_row_path_bilinear_sum():
     h.close()
 
 
+def test_row_path_tiny_matrices():
+    """Momentum-free row-path matrices with fewer rows than one chunk (1 to 5 rows; a stack
+    of one-row matrices): every tile is one ragged chunk."""
+    E = WL.TIER_EXPERT
+    specs = [WL.Spec("e1x4096", (1, 4096), E, expert=0), WL.Spec("e2x1024", (2, 1024), E, expert=1),
+             WL.Spec("e3x512", (3, 512), E, expert=2), WL.Spec("e5x2048", (5, 2048), E, expert=3),
+             WL.Spec("e3x1x1024", (3, 1, 1024), E)]
+    h = _harness(WL.Workload("tiny_rows", specs, WL.HP(), "normal", steps=3))
+    assert all(h.opt.info(k).rowpath == 1 for k in range(len(specs)))
+    for t in range(1, 4):
+        h.step(t, seed=11 * t)
+    h.close()
+
+
 def test_row_path_clamp_falls_back_to_phase_b():
     """eps = 1e-8 (App. A): the clamp binds at step 1, so the finalize queues the
     tensors for phase B and sum(U^2) is taken element by element."""
