@@ -1,29 +1,34 @@
 // Device kernels of libskewadam (sm_103a).
 //
-// One SkewAdam step (paper Sec. 3, Eq. 1, Algorithm 1). The work of a tensor is
-// four phases of tiles / items, each a grouped launch over an item table:
-//   A k_sumsq    : per-row and per-column sums of g^2 of a factored matrix
-//                  (Eq. 1): 16-byte bf16 loads issued eight rows at a time,
-//                  warp-shuffle row sums, column partials reduced across the CTA
-//                  in shared memory and written per row tile (no float atomics);
-//   F k_finalize : R <- b2 R + (1-b2) mean_c(G^2), C <- b2 C + (1-b2) mean_r(G^2),
-//                  1/sqrt(C_j) per column; the last item of a tensor forms mean(R);
-//   B k_rms      : the tier's momentum / exact second-moment update, U up to its
-//                  scalar coefficient and a compensated sum(U^2) per tile; the
-//                  last tile of a tensor forms RMS(U) and the clip factor
-//                  (Sec. 3 update clipping);
-//   C k_apply    : x = w (1 - lr*lambda) - lr*kappa*U in fp32 and the dithered
-//                  bf16 write-back with a Philox-4x32-10 counter hash.
+// One SkewAdam step (paper Sec. 3, Eq. 1, Algorithm 1) as seven grouped launches in
+// stream order, each over an item table of (tensor, tile) pairs:
+//   k_sumsq      phase A, strip tiles: per-row and per-column sums of g^2 of a
+//                factored matrix (Eq. 1), column partials per row tile (no atomics);
+//   k_rowsq      phase A, whole-row tiles of factored matrices 512 to 4096 wide:
+//                chunks of whole rows bulk-copied into a shared-memory ring; R_i
+//                formed in the tile (Eq. 1), per-column partials of g^2 and of
+//                g^2 / R_i (or M^2 / R_i after the momentum update, stored here),
+//                from which the finalize forms sum(U^2) by the bilinear identity;
+//   k_finalize   R / C moving averages (strip path) or C (row path), 1/sqrt(C_j),
+//                mean(R); on the row path also sum(U^2) and the clip factor, or the
+//                tensor is queued for phase B when the 1/sqrt(eps) clamp may bind;
+//   k_rms        phase B, strip and flat tiles: momentum / exact second-moment
+//                update, U up to its scalar and a compensated sum(U^2) per tile;
+//                the last tile forms RMS(U) and the clip factor (Sec. 3);
+//   k_fallback   phase B of the queued row-path tensors (element by element);
+//   k_apply      phase C, strip and flat tiles: x = w (1 - lr*lambda) - lr*kappa*U
+//                in fp32 and the dithered bf16 write-back (Philox-4x32-10);
+//   k_apply_rows phase C, whole-row tiles: the same on bulk-copied rows of W and
+//                G (or the new M).
 // The reconstructed second moment of a factored matrix is never formed:
 // 1/sqrt(max(R_i C_j / Rbar, eps)) = min(a_i * b_j, 1/sqrt(eps)) with
-// a_i = 1/sqrt(R_i / Rbar) per row and b_j = 1/sqrt(C_j) per column, both
-// computed once per tile into shared memory.
+// a_i = 1/sqrt(R_i / Rbar) per row and b_j = 1/sqrt(C_j) per column.
 //
-// The host launches the four phases over all tensors, each as one grouped
-// launch (phase-major). The per-step scalars are a kernel parameter (StepArgs,
-// constant bank). Values produced by an earlier phase of the same step are read
-// with L2-only (.cg) loads. When no element of a tile can reach the 1/sqrt(eps)
-// clamp (all but degenerate tiles), phase C takes a clamp-free path.
+// The per-step scalars are a kernel parameter (StepArgs, constant bank). Values
+// produced by an earlier launch of the same step are read with L2-only (.cg)
+// loads. When no element of a tile can reach the clamp (all but degenerate
+// tiles), phase C takes a clamp-free path. Every wait on a bulk copy is bounded
+// and reports a copy that does not land through the status word.
 #include <cuda_runtime.h>
 #include <type_traits>
 #include <stdint.h>
