@@ -16,9 +16,14 @@ Reported (one JSON line, rank 0):
                  of the 8 TB/s nominal and of the measured copy bandwidth;
   roofline    -- the dominant kernel's algorithmic bytes / its event-timed
                  duration against the measured HBM copy peak;
+  kernels_ms  -- each launch's mean event-timed duration;
+  step_spans  -- median / mean / min / max of the per-step times;
   e2e         -- the same metric through the C ABI with the gradients copied
-                 in from pinned host memory and the weights read back each step;
-  cpu_baseline-- the CPU oracle (single thread) on a bounded sample.
+                 in from pinned host memory and the weights read back each step
+                 (the step run as --e2e-groups handles over runs of consecutive
+                 tensors, so one group's copies overlap the others' steps);
+  cpu_baseline-- the CPU oracle (single thread) on a bounded sample;
+  clocks      -- SM clocks and throttle reasons sampled during the timed steps.
 Multi-GPU (torchrun): every rank updates its own full parameter set (the step
 has no cross-tensor coupling, so it shards by tensor with no collective);
 scaling is weak.
