@@ -302,8 +302,8 @@ int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t ndim, int64
                              uint32_t tensor_id, int64_t step, float lr, uint64_t seed, void *stream);
 
 /*
- * Kernel launches one skew_step performs (the step runs as one captured CUDA
- * graph of grouped launches; 0 for NULL or an empty handle).
+ * Kernel launches one skew_step performs (its grouped launches over item
+ * tables; 0 for NULL or an empty handle).
  */
 int64_t skew_launches_per_step(const skew_handle_t *h);
 
