@@ -288,18 +288,43 @@ const char *skew_kernel_name(int32_t k);
  * cudaStream_t. Updates weight and state in place, asynchronously on stream,
  * with the same kernels and results as skew_step on a one-tensor handle.
  *
- * The first call on a device looks up the array's device address with
- * cudaGetSymbolAddress (with that device current); make that first call before
- * any stream capture. All calls on a device share the one array: calls whose
+ * Every call looks up the array's device address on the current device with
+ * cudaGetSymbolAddress. The first such lookup on a device may load the
+ * library's device code there: make the first call on each device before any
+ * stream capture. All calls on a device share the one array: calls whose
  * work overlaps on the GPU (different streams, or other host threads) race
  * and corrupt each other's results -- serialise them. The array keeps the
  * last call's contents; everything a step needs zeroed is cleared by the step.
+ *
+ * Device-side failures: the whole-row kernels' bounded waits (as for
+ * skew_step) record a copy that did not land in a status word at the start of
+ * the array. No call clears it; skew_noalloc_sync_status reads it. A step
+ * whose wait gave up has left some tiles of that tensor unwritten.
  * Errors: SKEW_EINVAL (argument or state size), SKEW_ETOOBIG, SKEW_ECUDA.
  */
 #define SKEW_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
 int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t ndim, int64_t rows, int64_t cols, int32_t tier,
                              uint32_t flags, const skew_hparams_t *hp, void *state, size_t state_bytes,
                              uint32_t tensor_id, int64_t step, float lr, uint64_t seed, void *stream);
+
+/*
+ * Synchronises `stream` and reports the no-alloc status word of the current
+ * device: SKEW_OK, or SKEW_ETIMEOUT if a bounded device wait of a
+ * skew_step_tensor_noalloc call gave up since the word was last read (the word
+ * is then cleared, with a memset enqueued on `stream` and waited for). Uses no
+ * allocation (a 4-byte device-to-host copy). Errors: SKEW_ECUDA.
+ */
+int skew_noalloc_sync_status(void *stream);
+
+/*
+ * Self-test of that failure path: enqueues on `stream` one thread that waits,
+ * exactly as the whole-row kernels wait for a copied chunk, on an mbarrier
+ * phase that nothing completes; after its poll limit (about two seconds) the
+ * wait gives up and sets the no-alloc status word, so the next
+ * skew_noalloc_sync_status returns SKEW_ETIMEOUT. Nothing else is touched and
+ * the context stays usable. Asynchronous. Errors: SKEW_ECUDA.
+ */
+int skew_noalloc_selftest_wait_timeout(void *stream);
 
 /*
  * Kernel launches one skew_step performs (its grouped launches over item

@@ -556,6 +556,21 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity) {
     return false;
 }
 
+// After a wait gave up (status bit 2): one thread waits for chunks [c, issued_end) of a
+// ring of `stages` slots that are still in flight, so that the CTA does not leave while
+// a bulk copy may still write into its shared memory. Each gets up to eight more
+// rounds of polls (about sixteen seconds); a copy still outstanding after that is
+// recorded as status bit 4 and the CTA leaves anyway.
+__device__ __noinline__ void drain_copies(uint32_t *err, uint64_t *full, uint32_t stages, uint32_t c,
+                                          uint32_t issued_end) {
+    atomicOr(err, 2u);
+    for (uint32_t k = c; k < issued_end; ++k) {
+        bool landed = false;
+        for (int round = 0; round < 8 && !landed; ++round) landed = mbar_wait(&full[k % stages], (k / stages) & 1u);
+        if (!landed) atomicOr(err, 4u);
+    }
+}
+
 // Bulk copy global -> shared of `bytes` (multiple of 16, both ends 16-byte
 // aligned), completing on mbarrier `bar`, with an L2 eviction policy.
 __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar, uint64_t pol) {
@@ -821,15 +836,12 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         }
     }
     if (c < nch) {
-        // A chunk did not land in time: record it, give the copies in flight
-        // (chunks c .. issued) one more bounded wait each, and drop the tile.
-        // Issued so far: chunks [0, kRowStages) by the prologue and chunk k - 1 +
-        // kRowStages at each iteration k in [1, c); chunks before c have landed.
-        if (tid == 0) {
-            atomicOr(A.err, 2u);
-            const uint32_t issued_end = min(nch, c == 0 ? (uint32_t)kRowStages : c + kRowStages - 1);
-            for (uint32_t k = c; k < issued_end; ++k) (void)mbar_wait(&sm.full[k % kRowStages], (k / kRowStages) & 1u);
-        }
+        // A chunk did not land in time: record it, wait (bounded) for the copies in
+        // flight and drop the tile. Issued so far: chunks [0, kRowStages) by the
+        // prologue and chunk k - 1 + kRowStages at each iteration k in [1, c); chunks
+        // before c have landed.
+        if (tid == 0)
+            drain_copies(A.err, sm.full, kRowStages, c, min(nch, c == 0 ? (uint32_t)kRowStages : c + kRowStages - 1));
         return;
     }
     // per-tile partials, (sum of g^2, sum of g^2 / R_i) per column (the RPP threads that
@@ -953,6 +965,17 @@ __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem 
     if (j < T.m) {
         const float2 *p = T.pp + j;
         uint32_t r = sl;
+        // loads issued 32 (then 16) at a time ahead of the adds, which go in tile order
+        for (; r + 31 * tpc < T.rtiles; r += 32 * tpc) {
+            float2 v[32];
+#pragma unroll
+            for (int q = 0; q < 32; ++q) v[q] = __ldcg(p + int64_t(r + q * tpc) * T.m);
+#pragma unroll
+            for (int q = 0; q < 32; ++q) {
+                cs += v[q].x;
+                pa.add(v[q].y);
+            }
+        }
         for (; r + 15 * tpc < T.rtiles; r += 16 * tpc) {
             float2 v[16];
 #pragma unroll
@@ -1511,12 +1534,8 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
         }
         // every thread is done with slot st: refill it with chunk c + kRowStages
         if (__syncthreads_or(!ok)) {
-            if (tid == 0) {
-                atomicOr(A.err, 2u);
-                const uint32_t issued_end = min(nch, c + kRowStages);  // chunks [0, c + kRowStages) were issued
-                for (uint32_t k = c; k < issued_end; ++k)
-                    (void)mbar_wait(&sm.full[k % kRowStages], (k / kRowStages) & 1u);
-            }
+            if (tid == 0)  // chunks [0, c + kRowStages) were issued
+                drain_copies(A.err, sm.full, kRowStages, c, min(nch, c + kRowStages));
             return;
         }
         if (tid == 0 && c + kRowStages < nch) {
@@ -1755,11 +1774,8 @@ __device__ void rowsq_mom_tile(const StepArgs &A, const TensorDev &T, TensorScal
     }
     if (c < nch) {
         // a chunk did not land in time: as in rowsq_tile
-        if (tid == 0) {
-            atomicOr(A.err, 2u);
-            const uint32_t issued_end = min(nch, c == 0 ? (uint32_t)kMomStages : c + kMomStages - 1);
-            for (uint32_t k = c; k < issued_end; ++k) (void)mbar_wait(&sm.full[k % kMomStages], (k / kMomStages) & 1u);
-        }
+        if (tid == 0)
+            drain_copies(A.err, sm.full, kMomStages, c, min(nch, c == 0 ? (uint32_t)kMomStages : c + kMomStages - 1));
         return;
     }
     const int64_t base = int64_t(tile) * 8 * V;
@@ -1880,12 +1896,7 @@ __device__ void apply_rows_mom_body(const StepArgs &A, const TensorDev &T, uint3
         }
         // every thread is done with slot st: refill it with chunk c + kMomStages
         if (__syncthreads_or(!ok)) {
-            if (tid == 0) {
-                atomicOr(A.err, 2u);
-                const uint32_t issued_end = min(nch, c + kMomStages);
-                for (uint32_t k = c; k < issued_end; ++k)
-                    (void)mbar_wait(&sm.full[k % kMomStages], (k / kMomStages) & 1u);
-            }
+            if (tid == 0) drain_copies(A.err, sm.full, kMomStages, c, min(nch, c + kMomStages));
             return;
         }
         if (tid == 0 && c + kMomStages < nch) {

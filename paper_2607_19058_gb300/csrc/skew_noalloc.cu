@@ -12,13 +12,16 @@
 // process exits) and launches the same kernels as skew_step.
 //
 // The array's address is a device address that host code cannot name
-// directly: the host-side symbol is only a stand-in. It is looked up once per
-// device with cudaGetSymbolAddress, with that device current, on the first
-// call made on that device.
+// directly: the host-side symbol is only a stand-in. Every call looks it up
+// with cudaGetSymbolAddress for the current device (cheap once the module is
+// loaded; a cached address could go stale after cudaDeviceReset).
+//
+// The array's first bytes hold a status word of its own: the bounded waits of
+// the whole-row kernels set it when a copy does not land, every call leaves it
+// as it is, and skew_noalloc_sync_status reads and clears it.
 #include <cuda_runtime.h>
 
 #include <cmath>
-#include <mutex>
 
 #include "skew_plan.h"
 #include "skewadam.h"
@@ -28,10 +31,16 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_scratch[SKEW_NOALLOC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-unsigned char *g_scratch_ptr[kMaxDevices] = {};
+// Offset of the status word in the array (kept apart from any call's scratch layout).
+constexpr size_t kErrOffset = 0;
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// The array's device address on the current device, or null.
+unsigned char *scratch_base() {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess) return nullptr;
+    return static_cast<unsigned char *>(p);
+}
 
 struct SetupTables {
     uint2 *A;
@@ -123,10 +132,10 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     const uint32_t nB = row ? 0 : G.ntiles, nC = row ? 0 : G.ntiles, nCR = row ? G.rtiles : 0;
 
     // ---- scratch layout inside the fixed array --------------------------------------
-    size_t off = 0;
+    size_t off = align256(kErrOffset + 16);  // the status word comes first
     const size_t o_scal = off;   off = align256(off + sizeof(TensorScal));
     const size_t o_fb = off;     off = align256(off + 8);
-    const size_t o_err = off;    off = align256(off + 16);
+    const size_t o_err = kErrOffset;
     const size_t o_tens = off;   off = align256(off + sizeof(TensorDev));
     const size_t o_iA = off;     off = align256(off + sizeof(uint2) * nA);
     const size_t o_iR = off;     off = align256(off + sizeof(uint2) * nR);
@@ -151,22 +160,12 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     const size_t o_u2 = off;     off = align256(off + 8 * size_t(G.ntiles));
     if (off > SKEW_NOALLOC_SCRATCH_BYTES) return SKEW_ETOOBIG;  // too large for the fixed array
 
-    // ---- device address of the fixed array, once per device ------------------------
+    // ---- device address of the fixed array on the current device ---------------------
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return SKEW_ECUDA;
-    if (dev < 0 || dev >= kMaxDevices) return SKEW_EINVAL;
-    unsigned char *base;
-    {
-        std::lock_guard<std::mutex> lk(g_mu);
-        if (!g_scratch_ptr[dev]) {
-            void *p = nullptr;
-            e = cudaGetSymbolAddress(&p, g_scratch);
-            if (e != cudaSuccess || !p) return SKEW_ECUDA;  // the array's device address is unknown
-            g_scratch_ptr[dev] = static_cast<unsigned char *>(p);
-        }
-        base = g_scratch_ptr[dev];
-    }
+    unsigned char *const base = scratch_base();
+    if (!base) return SKEW_ECUDA;  // the array's device address is unknown
 
     TensorDev td{};
     td.w = (uint16_t *)weight;
@@ -260,4 +259,25 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     e = (cudaError_t)launch_phases(a, lp, stream, nullptr);
     if (e != cudaSuccess) return SKEW_ECUDA;
     return SKEW_OK;
+}
+
+extern "C" int skew_noalloc_sync_status(void *stream) {
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return SKEW_ECUDA;
+    unsigned char *const base = scratch_base();
+    if (!base) return SKEW_ECUDA;
+    uint32_t word = 0;
+    if (cudaMemcpy(&word, base + kErrOffset, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return SKEW_ECUDA;
+    if (!word) return SKEW_OK;
+    if (cudaMemsetAsync(base + kErrOffset, 0, 4, s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
+        return SKEW_ECUDA;
+    return SKEW_ETIMEOUT;
+}
+
+extern "C" int skew_noalloc_selftest_wait_timeout(void *stream) {
+    unsigned char *const base = scratch_base();
+    if (!base) return SKEW_ECUDA;
+    return launch_wait_selftest(reinterpret_cast<uint32_t *>(base + kErrOffset), stream) == (int)cudaSuccess
+               ? SKEW_OK
+               : SKEW_ECUDA;
 }

@@ -29,7 +29,8 @@ KIND_FULL, KIND_FACTORED = 0, 1
 EXPORTS = ["skew_create", "skew_destroy", "skew_state_bytes", "skew_workspace_bytes", "skew_bind", "skew_step",
            "skew_sync_status", "skew_tensor_scalars", "skew_matrix_scalars", "skew_tensor_info", "skew_num_tensors", "skew_last_error",
            "skew_profile_begin", "skew_profile_end", "skew_kernel_name", "skew_step_tensor_noalloc",
-           "skew_launches_per_step", "skew_selftest_wait_timeout"]
+           "skew_launches_per_step", "skew_selftest_wait_timeout", "skew_noalloc_sync_status",
+           "skew_noalloc_selftest_wait_timeout"]
 
 
 class SkewError(RuntimeError):
@@ -108,6 +109,10 @@ def load(path: Optional[str] = None) -> C.CDLL:
         L.skew_step_tensor_noalloc.argtypes = [vp, vp, i32, i64, i64, i32, C.c_uint32, C.POINTER(HParams), vp, sz,
                                                C.c_uint32, i64, C.c_float, u64, vp]
         L.skew_step_tensor_noalloc.restype = C.c_int
+        L.skew_noalloc_sync_status.argtypes = [vp]
+        L.skew_noalloc_sync_status.restype = C.c_int
+        L.skew_noalloc_selftest_wait_timeout.argtypes = [vp]
+        L.skew_noalloc_selftest_wait_timeout.restype = C.c_int
         if path is None:
             _lib = L
         return L
@@ -217,6 +222,22 @@ def skew_step_tensor_noalloc(weight_ptr: int, grad_ptr: int, ndim: int, rows: in
         why = {SKEW_EINVAL: "invalid argument or state size", SKEW_ECUDA: "CUDA error",
                SKEW_ETOOBIG: f"tensor needs more than the {NOALLOC_SCRATCH_BYTES} bytes of fixed scratch"}
         raise SkewError(rc, why.get(rc, "error"))
+
+
+def skew_noalloc_sync_status(stream: int) -> None:
+    """Synchronises `stream`; raises SkewError(SKEW_ETIMEOUT) once if a bounded device wait of a
+    no-alloc call gave up since the last read (the status word is then cleared)."""
+    rc = load().skew_noalloc_sync_status(stream)
+    if rc != SKEW_OK:
+        why = {SKEW_ETIMEOUT: "a bounded device wait of a no-alloc step gave up", SKEW_ECUDA: "CUDA error"}
+        raise SkewError(rc, why.get(rc, "error"))
+
+
+def skew_noalloc_selftest_wait_timeout(stream: int) -> None:
+    """Makes one bounded device wait run out against the no-alloc status word."""
+    rc = load().skew_noalloc_selftest_wait_timeout(stream)
+    if rc != SKEW_OK:
+        raise SkewError(rc, "CUDA error")
 
 
 def hparams(beta1=0.9, beta2=0.999, eps=1e-8, clip_d=1.0, weight_decay=0.05, policy=POLICY_TIERED) -> HParams:

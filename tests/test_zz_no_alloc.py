@@ -8,7 +8,9 @@ scratch is a fixed array inside the library instead of a caller workspace.
 Checked through the C ABI against the regular path (skew_create / skew_bind /
 skew_step on a one-tensor handle) on two consecutive steps, for a factored
 expert matrix, a momentum backbone matrix, the router's exact second moment
-and a backbone vector. The file is named so that pytest collects it last.
+and a backbone vector; and its status word: a bounded device wait that gives
+up is reported once by skew_noalloc_sync_status, after which the entry point
+keeps stepping in parity. The file is named so that pytest collects it last.
 """
 import ctypes as C
 
@@ -21,9 +23,12 @@ from paper_2607_19058_gb300 import workloads as WL
 pytestmark = pytest.mark.gpu
 
 # (8192, 4096) expert: a momentum-free matrix on the whole-row path; (50304, 4096)
-# backbone: the paper's embedding, the largest tensor the fixed scratch is sized for.
+# backbone: the paper's embedding, the largest tensor the fixed scratch is sized for;
+# (4096, 4096) and (3001, 2048) experts: matrices that skew_step runs in its pipelined
+# launch, which the no-alloc entry point must match with the separate launches.
 SHAPES = [((300, 1000), S.TIER_EXPERT), ((517, 136), S.TIER_BACKBONE), ((4096, 127), S.TIER_ROUTER),
-          ((100003,), S.TIER_BACKBONE), ((8192, 4096), S.TIER_EXPERT), ((50304, 4096), S.TIER_BACKBONE)]
+          ((100003,), S.TIER_BACKBONE), ((8192, 4096), S.TIER_EXPERT), ((50304, 4096), S.TIER_BACKBONE),
+          ((4096, 4096), S.TIER_EXPERT), ((3001, 2048), S.TIER_EXPERT)]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -93,3 +98,39 @@ def test_noalloc_fp32_matches_regular_path():
             assert torch.equal(w_ref, w_na), f"fp32 weights differ at step {t}"
             assert torch.equal(ref.state[:nbytes].view(torch.float32), state)
         ref.close()
+
+
+def test_noalloc_reports_a_timed_out_wait_once_then_steps_in_parity():
+    """The self-test makes one bounded wait give up against the no-alloc status word (no
+    fault: an mbarrier phase that nothing completes). The next skew_noalloc_sync_status
+    reports SKEW_ETIMEOUT and clears the word; a read after that is clean, and whole-row
+    steps through the entry point keep matching the regular path bit for bit."""
+    dev = torch.device("cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    S.skew_noalloc_sync_status(stream)            # whatever an earlier test left is cleared
+    shape, tier = (8192, 4096), S.TIER_EXPERT
+    torch.manual_seed(3)
+    w0 = (torch.randn(shape, device=dev) * 0.02).to(torch.bfloat16)
+    g = torch.empty(shape, dtype=torch.bfloat16, device=dev)
+    hp = S.hparams(0.9, 0.999, 1e-30, 1.0, 0.1, S.POLICY_TIERED)
+    w_ref, w_na = w0.clone(), w0.clone()
+    ref = S.SkewAdam([(w_ref, g, tier)], hp)
+    nbytes = ref.state_bytes
+    state = torch.zeros(nbytes // 4, dtype=torch.float32, device=dev)
+    S.skew_noalloc_selftest_wait_timeout(stream)
+    for t in (1, 2):
+        g.copy_((torch.randn(shape, device=dev) * 1e-3).to(torch.bfloat16))
+        ref.step(t, 1e-3, 91)
+        S.skew_step_tensor_noalloc(w_na.data_ptr(), g.data_ptr(), 2, shape[0], shape[1], tier, 0, hp,
+                                   state.data_ptr(), nbytes, 0, t, 1e-3, 91, stream)
+        if t == 1:
+            with pytest.raises(S.SkewError) as e:
+                S.skew_noalloc_sync_status(stream)
+            assert e.value.code == S.SKEW_ETIMEOUT
+            S.skew_noalloc_sync_status(stream)    # reported once: the word is clear again
+        torch.cuda.synchronize()
+        assert torch.equal(w_ref.view(torch.int16), w_na.view(torch.int16)), f"weights differ at step {t}"
+        assert torch.equal(ref.state[:nbytes].view(torch.float32), state), f"state differs at step {t}"
+    S.skew_noalloc_sync_status(stream)
+    ref.sync_status()
+    ref.close()
