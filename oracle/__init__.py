@@ -52,7 +52,8 @@ class _Tensor(C.Structure):
 
 class _HParams(C.Structure):
     _fields_ = [("beta1", C.c_double), ("beta2", C.c_double), ("eps", C.c_double),
-                ("clip_d", C.c_double), ("weight_decay", C.c_double), ("annealed", C.c_int32)]
+                ("clip_d", C.c_double), ("weight_decay", C.c_double), ("annealed", C.c_int32),
+                ("gscale", C.c_double)]
 
 
 def lib():
@@ -150,11 +151,13 @@ class TensorState:
         return sum(a.nbytes for a in (self.M, self.v, self.R, self.C) if a is not None)
 
 
-def hparams(beta1, beta2, eps, clip_d, weight_decay, annealed: bool = False):
+def hparams(beta1, beta2, eps, clip_d, weight_decay, annealed: bool = False, gscale: float = 1.0):
     """The fp32 hyper-parameters widened to double (both sides use the fp32 values).
-    `annealed`: the Adafactor comparator's decay 1 - t^-0.8 without bias correction."""
+    `annealed`: the Adafactor comparator's decay 1 - t^-0.8 without bias correction.
+    `gscale`: the trainer's global gradient-norm clip factor of the step (an fp32 value):
+    the step sees gscale * G."""
     f = lambda x: float(np.float32(x))
-    return _HParams(f(beta1), f(beta2), f(eps), f(clip_d), f(weight_decay), int(annealed))
+    return _HParams(f(beta1), f(beta2), f(eps), f(clip_d), f(weight_decay), int(annealed), f(gscale))
 
 
 def tensor_step(w_bits: np.ndarray, g_bits: np.ndarray, st: TensorState, tid: int, hp, step: int,

@@ -249,6 +249,9 @@ typedef struct {
     double beta1, beta2, eps, clip_d, weight_decay;
     int32_t annealed;   /* 1: the Adafactor comparator's decay beta2_t = 1 - t^-0.8 */
                         /* (as an fp32 value) and no bias correction; beta2 unused  */
+    double gscale;      /* the trainer's global gradient-norm clip factor of this   */
+                        /* step (Sec. 4 training setup, App. A Table 9: clip 1.0):  */
+                        /* the step sees gscale * G, formed in fp64; 1 = no clip    */
 } so_hparams_t;
 
 /*
@@ -280,7 +283,7 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
     /* Second moment: full (Algorithm 1, full branch) or factored (Eq. 1). */
     if (T->kind == SO_KIND_FULL) {
         for (int64_t e = 0; e < numel; ++e) {
-            double g = so_grad(T, e);
+            double g = hp->gscale * so_grad(T, e);
             T->v[e] = (float)(b2 * (double)T->v[e] + (1.0 - b2) * g * g);
         }
     } else {
@@ -289,7 +292,7 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
         if (!rs || !cs) { free(rs); free(cs); free(U); return -1; }
         for (int64_t i = 0; i < n; ++i)
             for (int64_t j = 0; j < m; ++j) {
-                double g = so_grad(T, i * m + j);
+                double g = hp->gscale * so_grad(T, i * m + j);
                 rs[i] += g * g;
                 cs[j] += g * g;
             }
@@ -308,7 +311,7 @@ int so_tensor_step(const so_tensor_t *T, const so_hparams_t *hp, int64_t t, doub
     for (int64_t i = 0; i < n; ++i)
         for (int64_t j = 0; j < m; ++j) {
             const int64_t e = i * m + j;
-            double g = so_grad(T, e);
+            double g = hp->gscale * so_grad(T, e);
             double vhat;
             if (T->kind == SO_KIND_FULL)
                 vhat = (double)T->v[e];

@@ -55,8 +55,8 @@ class Brute:
         self.R = z(self.n) if kind == O.KIND_FACTORED else None
         self.C = z(self.m) if kind == O.KIND_FACTORED else None
 
-    def step(self, w_bits, g_bits, t, lr, seed, tid, b1, b2, eps, d, lam):
-        G = _f(g_bits).astype(np.float64).reshape(self.n, self.m)
+    def step(self, w_bits, g_bits, t, lr, seed, tid, b1, b2, eps, d, lam, gscale=1.0):
+        G = gscale * _f(g_bits).astype(np.float64).reshape(self.n, self.m)
         Wt = _f(w_bits).astype(np.float64).reshape(self.n, self.m)
         G2 = G * G
         rbar = 0.0
@@ -103,12 +103,16 @@ def _ulps(a, b):
 
 
 @pytest.mark.parametrize("shape,tier,policy", CASES)
-@pytest.mark.parametrize("eps,lr,lam", [(1e-30, 1e-3, 0.1), (1e-8, 3e-4, 0.05)])
-def test_oracle_matches_brute_force(shape, tier, policy, eps, lr, lam):
+@pytest.mark.parametrize("eps,lr,lam,gscale", [(1e-30, 1e-3, 0.1, 1.0), (1e-8, 3e-4, 0.05, 1.0),
+                                               (1e-30, 1e-3, 0.1, 0.37)])
+def test_oracle_matches_brute_force(shape, tier, policy, eps, lr, lam, gscale):
+    """`gscale` is the trainer's global gradient-norm clip factor of the step (Sec. 4 training
+    setup, App. A Table 9): the brute force forms gscale * G and steps on it."""
     rng = np.random.default_rng(hash((shape, tier, policy, eps)) & 0xFFFF)
     b1, b2 = float(F32(0.9)), float(F32(0.999))
     eps32, lr32, lam32, d32 = float(F32(eps)), float(F32(lr)), float(F32(lam)), float(F32(0.5))
-    hp = O.hparams(0.9, 0.999, eps, 0.5, lam)
+    gs32 = float(F32(gscale))
+    hp = O.hparams(0.9, 0.999, eps, 0.5, lam, gscale=gscale)
     st = O.TensorState(shape, tier, policy)
     br = Brute(shape, st.kind, st.momentum, st.decay)
     numel = int(np.prod(shape))
@@ -121,7 +125,7 @@ def test_oracle_matches_brute_force(shape, tier, policy, eps, lr, lam):
         if t == 5:
             g[: max(1, numel // 3)] = 0
         o = O.tensor_step(w, g, st, tid, hp, t, lr32, seed, want_x=True)
-        bw, bx, brr, bs = br.step(wb, g, t, lr32, seed, tid, b1, b2, eps32, d32, lam32)
+        bw, bx, brr, bs = br.step(wb, g, t, lr32, seed, tid, b1, b2, eps32, d32, lam32, gs32)
         for k in ("M", "v", "R", "C"):
             a, b = getattr(st, k), getattr(br, k)
             if a is not None:

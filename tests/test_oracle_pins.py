@@ -526,3 +526,76 @@ def test_nx1_and_1xm_factored_exact():
         # decay differs between tiers (router exempt); U and its RMS do not
         for a, b in zip(of, ov):
             assert abs(a["rms"] - b["rms"]) <= 1e-6 * b["rms"]
+
+
+# --------------------------------------------------------------------------
+# The trainer's global gradient-norm clip (Sec. 4 training setup, App. A Table 9:
+# clip 1.0) applied as a per-step scale gamma of the gradient the step sees
+# --------------------------------------------------------------------------
+def _hp_g(gscale, **kw):
+    return O.hparams(0.9, 0.999, kw.get("eps", 1e-30), 1.0, kw.get("wd", 0.1), gscale=gscale)
+
+
+def test_gscale_power_of_two_equals_halved_gradient():
+    """gamma = 0.5 is the same step, bit for bit, as gamma = 1 on a gradient halved
+    exactly in bf16 (a power-of-two scale of a normal bf16 value is exact), on every
+    tier and over three steps, so every place the gradient enters takes gamma."""
+    rng = np.random.default_rng(41)
+    for shape, tier in (((33, 17), O.TIER_EXPERT), ((20, 40), O.TIER_BACKBONE), ((16, 8), O.TIER_ROUTER),
+                        ((129,), O.TIER_BACKBONE)):
+        w = _bf16(rng.normal(0, 0.02, shape).astype(np.float32)).reshape(-1)
+        gs = [_bf16(rng.normal(0, 1e-3, shape).astype(np.float32)).reshape(-1) for _ in range(3)]
+        half = [_bf16(_f(g) * np.float32(0.5)) for g in gs]
+        assert all(np.array_equal(_f(h).astype(np.float64), 0.5 * _f(g).astype(np.float64)) for h, g in zip(half, gs))
+        sa, sb = O.TensorState(shape, tier), O.TensorState(shape, tier)
+        wa, wb = w.copy(), w.copy()
+        for t in (1, 2, 3):
+            oa = O.tensor_step(wa, gs[t - 1], sa, 3, _hp_g(0.5), t, 1e-3, 17, want_x=True)
+            ob = O.tensor_step(wb, half[t - 1], sb, 3, _hp_g(1.0), t, 1e-3, 17, want_x=True)
+            assert np.array_equal(oa["x"].view(np.uint32), ob["x"].view(np.uint32)), (shape, t)
+            assert np.array_equal(wa, wb)
+            for key in ("M", "v", "R", "C"):
+                if getattr(sa, key) is not None:
+                    assert np.array_equal(getattr(sa, key), getattr(sb, key)), (shape, t, key)
+
+
+def test_gscale_step1_full_v_leaves_sign_and_is_not_a_learning_rate():
+    """Algorithm 1, full v at t = 1: U = sign(g) whatever gamma > 0 (v = (1-b2) gamma^2 g^2),
+    so the step's weights do not depend on gamma; scaling the learning rate by gamma
+    instead changes them. The clip factor therefore cannot be folded into lr."""
+    rng = np.random.default_rng(42)
+    shape = (64, 8)
+    g = _bf16(rng.normal(0, 1e-3, shape).astype(np.float32)).reshape(-1)
+    w = _bf16(rng.normal(0, 0.02, shape).astype(np.float32)).reshape(-1)
+    lr, gam = float(F32(1e-3)), float(F32(0.37))
+    for tier, shp in ((O.TIER_ROUTER, shape), (O.TIER_BACKBONE, (512,))):
+        outs = {}
+        for key, gscale, lr_k in (("one", 1.0, lr), ("gamma", gam, lr), ("lr", 1.0, lr * gam)):
+            st = O.TensorState(shp, tier)
+            ww = w.copy()
+            outs[key] = (O.tensor_step(ww, g, st, 0, _hp_g(gscale), 1, lr_k, 9, want_x=True), ww, st)
+        assert np.array_equal(outs["one"][1], outs["gamma"][1])             # weights unchanged by gamma
+        assert not np.array_equal(outs["one"][1], outs["lr"][1])            # but changed by lr * gamma
+        assert np.allclose(outs["gamma"][2].v, gam * gam * outs["one"][2].v, rtol=2e-7, atol=0)
+        if tier == O.TIER_BACKBONE:
+            assert np.allclose(outs["gamma"][2].M, gam * outs["one"][2].M, rtol=2e-7, atol=0)
+
+
+def test_gscale_second_step_is_not_scale_invariant():
+    """With a history the EMAs mix steps seen at different scales: a gradient scaled at
+    step 2 only (zero at step 1 leaves v = 0, so take g at both steps) changes the step
+    on every tier, factored experts included."""
+    rng = np.random.default_rng(43)
+    shape = (24, 32)
+    g1 = _bf16(rng.normal(0, 1e-3, shape).astype(np.float32)).reshape(-1)
+    g2 = _bf16(rng.normal(0, 1e-3, shape).astype(np.float32)).reshape(-1)
+    w = _bf16(rng.normal(0, 0.02, shape).astype(np.float32)).reshape(-1)
+    for tier in (O.TIER_EXPERT, O.TIER_BACKBONE, O.TIER_ROUTER):
+        res = []
+        for gam2 in (1.0, 0.37):
+            st = O.TensorState(shape, tier)
+            ww = w.copy()
+            O.tensor_step(ww, g1, st, 0, _hp_g(1.0), 1, 1e-3, 9)
+            o = O.tensor_step(ww, g2, st, 0, _hp_g(gam2), 2, 1e-3, 9, want_x=True)
+            res.append(o["x"])
+        assert np.max(np.abs(res[0].astype(np.float64) - res[1].astype(np.float64))) > 1e-6
