@@ -62,6 +62,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="target oracle time of the CPU baseline sample")
     p.add_argument("--ref-seconds", type=float, default=150.0, help="target total time of --impl reference")
+    p.add_argument("--grad-scale", type=float, default=None,
+                   help="step on gamma * G with gamma a device scalar (the trainer's global-norm clip inside the step)")
     return p.parse_args()
 
 
@@ -397,12 +399,13 @@ def run_ours(args):
     bm = byte_model(opt, len(wl.specs))
     wg_bytes = sum(w.numel() * w.element_size() + g.numel() * g.element_size() for w, g in zip(W, G))
     stream = torch.cuda.current_stream()
+    gscale = None if args.grad_scale is None else torch.tensor([args.grad_scale], dtype=torch.float32, device=dev)
     torch.cuda.synchronize()
 
     step = 0
     for _ in range(args.warmup):
         step += 1
-        opt.step(step, hp.lr, args.seed)
+        opt.step(step, hp.lr, args.seed, grad_scale=gscale)
     opt.sync_status()
     if world > 1:
         dist.barrier()
@@ -415,7 +418,7 @@ def run_ours(args):
     e0.record(stream)
     for i in range(args.steps):
         step += 1
-        opt.step(step, hp.lr, args.seed)
+        opt.step(step, hp.lr, args.seed, grad_scale=gscale)
         marks[i + 1].record(stream)
     torch.cuda.synchronize()
     clocks = clocks_stop(clk)
@@ -534,7 +537,8 @@ def run_ours(args):
             "config": {"workload": wl.name, "params": bm["N"], "tensors": len(wl.specs), "policy": policy_name(wl),
                        "state_bytes": opt.state_bytes, "workspace_bytes": opt.workspace_bytes,
                        "l2": f"inputs larger than L2 ({wg_bytes / 1e9:.1f} GB of weights + grads vs 129 MiB), no flush",
-                       "weights_grads": "bf16, W~N(0,0.02^2), G~N(0,1e-3^2)"},
+                       "weights_grads": "bf16, W~N(0,0.02^2), G~N(0,1e-3^2)",
+                       "grad_scale": args.grad_scale},
             "hbm": {"min_bytes_per_step": bm["step_min"], "achieved_gbs": step_gbs,
                     "frac_of_8tbs": step_gbs / NOMINAL_HBM_GBS, "frac_of_measured": step_gbs / peak,
                     "peak_gbs": peak, "peak_source": peak_src},

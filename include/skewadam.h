@@ -212,6 +212,26 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
 int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *stream);
 
 /*
+ * skew_step with the trainer's global gradient-norm clip applied inside the step.
+ * The paper's training setup (Sec. 4) and App. A Table 9 clip the global gradient
+ * norm at 1.0 before the optimizer step: G <- gamma * G with gamma = min(1, c /
+ * ||G||). Here the step sees gamma * G without a separate pass over the gradients:
+ * gamma enters only the moving-average increments ((1 - beta1) gamma on g,
+ * (1 - beta2) gamma^2 on g^2) and the update coefficient of momentum-free tensors,
+ * so the step reads and writes exactly the bytes of skew_step. (Scaling the learning
+ * rate instead is not the same step: the second moments are moving averages of the
+ * scaled gradient.)
+ *   grad_scale : device pointer to one fp32 gamma (finite), computed by the caller
+ *                on `stream` before this call (e.g. from its norm reduction); read
+ *                by the kernels, never by the host; 4-byte aligned. NULL means
+ *                gamma = 1, and then the call is skew_step, bit for bit; so is a
+ *                pointer to 1.0f.
+ * Other arguments, asynchrony and errors as skew_step (SKEW_EINVAL also for a
+ * misaligned grad_scale).
+ */
+int skew_step_scaled(skew_handle_t *h, int64_t step, float lr, uint64_t seed, const float *grad_scale, void *stream);
+
+/*
  * Synchronises `stream` and reports the device-side status word of the last
  * steps: SKEW_OK, or SKEW_ETIMEOUT if a bounded device wait gave up (the word
  * is cleared by this call). Errors: SKEW_ESTATE, SKEW_ECUDA.

@@ -423,7 +423,12 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
 }
 
 int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *stream) {
+    return skew_step_scaled(h, step, lr, seed, nullptr, stream);
+}
+
+int skew_step_scaled(skew_handle_t *h, int64_t step, float lr, uint64_t seed, const float *grad_scale, void *stream) {
     if (!h) return SKEW_EINVAL;
+    if ((uintptr_t)grad_scale & 3) return fail(h, SKEW_EINVAL, "grad_scale must be a 4-byte aligned device pointer");
     if (!h->bound) return fail(h, SKEW_ESTATE, "skew_step before skew_bind");
     if (step < 1) return fail(h, SKEW_EINVAL, "step must be >= 1 (got %lld)", (long long)step);
     if (!std::isfinite(lr) || lr < 0.f) return fail(h, SKEW_EINVAL, "lr must be finite and >= 0");
@@ -450,6 +455,7 @@ int skew_step(skew_handle_t *h, int64_t step, float lr, uint64_t seed, void *str
     a.step_lo = (uint32_t)(uint64_t)step;
     a.seed_lo = (uint32_t)seed;
     a.seed_hi = (uint32_t)(seed >> 32);
+    a.gscale = grad_scale;
 
     cudaEvent_t *ev = nullptr;
     if (h->prof_used < h->prof_max) {

@@ -213,6 +213,23 @@ __device__ __forceinline__ uint32_t sr_bf16(float x, uint32_t r) {
     return (b + r) >> 16;
 }
 
+// The gradient scale gamma of the step (the trainer's global gradient-norm clip, Sec. 4
+// training setup, App. A Table 9): the step sees gamma * G. It enters only through the
+// moving-average increments, (1 - beta2) gamma^2 on g^2 and (1 - beta1) gamma on g, and
+// the update coefficient of momentum-free tensors (U = coef * gamma * g / D; set_clip),
+// so no kernel reads the gradient more than without it. With gamma = 1 every product
+// below is exact and the step is bit for bit the unscaled one.
+struct GScale {
+    float c1, c2;  // (1 - beta1) gamma, (1 - beta2) gamma^2
+    float gam;
+};
+
+__device__ __forceinline__ GScale grad_scale(const StepArgs &A) {
+    if (!A.gscale) return GScale{A.c1, A.c2, 1.f};
+    const float g = __ldg(A.gscale);
+    return GScale{A.c1 * g, A.c2 * (g * g), g};
+}
+
 // a_i = 1/sqrt(R_i / Rbar), with Rbar = rbar_s * 2^-rbar_e (rbar_s in [1,2)); +inf if Rbar == 0.
 __device__ __forceinline__ float row_scale(float Ri, float rbar_s, int rbar_e) {
     if (rbar_s == 0.f) return __int_as_float(0x7F800000);
@@ -719,7 +736,7 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
         for (uint32_t c = 0; c < nch && c < (uint32_t)kRowStages; ++c) row_issue(T, tile, c, sm, pol);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const float b2 = A.b2, c2 = A.c2, inv_m = 1.0f / (float)(8 * V);  // m is a power of two: exact
+    const float b2 = A.b2, c2 = grad_scale(A).c2, inv_m = 1.0f / (float)(8 * V);  // m is a power of two: exact
     // per column pair: sums of g^2, the compensated (hi, lo) sum of g^2 / R_i and its open fp32 part
     float2 cs[NV][4], ph[NV][4], pl[NV][4], t[NV][4];
 #pragma unroll
@@ -933,7 +950,8 @@ __device__ void set_rbar(TensorScal &S, double rbar) {
 // From s = sum of (U / coef)^2: sum(U^2), RMS(U), the clip factor
 // kappa = 1 / max(1, RMS / d) (Sec. 3 update clipping) and lr * kappa * coef.
 __device__ void set_clip(const StepArgs &A, const TensorDev &T, TensorScal &S, double s) {
-    const double coef = T.momentum ? A.coef_mom : A.coef_plain;
+    // a momentum-free tensor's U is coef * gamma * g / D (M already carries gamma)
+    const double coef = T.momentum ? A.coef_mom : A.coef_plain * (double)grad_scale(A).gam;
     const double su2 = s * coef * coef;
     const double rms = sqrt(su2 / (double)T.numel);
     const double kappa = 1.0 / fmax(1.0, rms / (double)A.clip_d);
@@ -1009,7 +1027,7 @@ __device__ void phase_F_row(const StepArgs &A, uint32_t t, uint32_t local, Smem 
         }
         const float P = pair_f(pa.hi, pa.lo);
         const float mean = __fdiv_rn(cs, (float)T.n);
-        const float Cn = fmaf(A.b2, Cold, A.c2 * mean);
+        const float Cn = fmaf(A.b2, Cold, grad_scale(A).c2 * mean);
         T.C[j] = Cn;
         T.bsc[j] = __frsqrt_rn(Cn);
         if (P > 0.f) {
@@ -1096,7 +1114,7 @@ __device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm)
         if (threadIdx.x < kFinChunk && i < T.n) {
             const float rs = strided_sum(T.rowp + i, T.n, T.strips);
             const float mean = __fdiv_rn(rs, (float)T.m);
-            const float Rn = fmaf(A.b2, T.R[i], A.c2 * mean);
+            const float Rn = fmaf(A.b2, T.R[i], grad_scale(A).c2 * mean);
             T.R[i] = Rn;
             rd = (double)Rn;
         }
@@ -1107,7 +1125,7 @@ __device__ void phase_F(const StepArgs &A, uint32_t t, uint32_t local, Smem &sm)
         if (threadIdx.x < kFinChunk && j < T.m) {
             const float cs = strided_sum(T.colp + j, T.m, T.rowtiles);
             const float mean = __fdiv_rn(cs, (float)T.n);
-            const float Cn = fmaf(A.b2, T.C[j], A.c2 * mean);
+            const float Cn = fmaf(A.b2, T.C[j], grad_scale(A).c2 * mean);
             T.C[j] = Cn;
             T.bsc[j] = __frsqrt_rn(Cn);
         }
@@ -1145,7 +1163,7 @@ __device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
     float *__restrict__ M_ = T.M;
     const int64_t n = T.n, m = T.m, row0 = F.row0, RG = F.RG, col0 = F.col0;
     const int valid = F.valid;
-    const float b1 = A.b1, c1 = A.c1, ce = A.ce;
+    const float b1 = A.b1, c1 = grad_scale(A).c1, ce = A.ce;
     const bool mnew = MOM && T.rowpath;  // phase B of a queued row-path tensor: M is already new
     const float *rows = meta.rows + F.rg;
     float b[8];
@@ -1216,6 +1234,7 @@ __device__ Acc2 rms_fact_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
 
 template <bool VEC>
 __device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t tile, const Pol &pol) {
+    const GScale gsc = grad_scale(A);
     Acc2 acc;
     for (int k = 0; k < kFlatVecPerThread; ++k) {
         const int64_t e0 = 8 * (int64_t(tile) * kThreads * kFlatVecPerThread + int64_t(k) * kThreads + threadIdx.x);
@@ -1228,13 +1247,13 @@ __device__ Acc2 rms_full_tile(const StepArgs &A, const TensorDev &T, uint32_t ti
             load8_elem(T.g, T.f32, e0, valid, g);
         load_f8<VEC>(T.v + e0, valid, v, false);
 #pragma unroll
-        for (int c = 0; c < 8; ++c) v[c] = fmaf(A.b2, v[c], A.c2 * (g[c] * g[c]));
+        for (int c = 0; c < 8; ++c) v[c] = fmaf(A.b2, v[c], gsc.c2 * (g[c] * g[c]));
         store_f8<VEC>(T.v + e0, valid, v);
         if (T.momentum) {
             float mm[8];
             load_f8<VEC>(T.M + e0, valid, mm, false);
 #pragma unroll
-            for (int c = 0; c < 8; ++c) y[c] = fmaf(A.b1, mm[c], A.c1 * g[c]);
+            for (int c = 0; c < 8; ++c) y[c] = fmaf(A.b1, mm[c], gsc.c1 * g[c]);
             store_f8<VEC>(T.M + e0, valid, y);
         } else {
 #pragma unroll
@@ -1666,7 +1685,8 @@ __device__ void rowsq_mom_tile(const StepArgs &A, const TensorDev &T, TensorScal
         for (uint32_t c = 0; c < nch && c < (uint32_t)kMomStages; ++c) mom_issue(T, T.g, tile, c, sm.buf, sm.full, pol);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const float b1 = A.b1, c1 = A.c1, b2 = A.b2, c2 = A.c2, inv_m = 1.0f / (float)(8 * V);  // exact
+    const GScale gsc = grad_scale(A);
+    const float b1 = A.b1, c1 = gsc.c1, b2 = A.b2, c2 = gsc.c2, inv_m = 1.0f / (float)(8 * V);  // exact
     const float2 b12 = make_float2(b1, b1), c12 = make_float2(c1, c1);
     // per column pair: sums of g^2, the compensated (hi, lo) sum of M^2 / R_i and its open fp32 part
     float2 cs[NV][4], ph[NV][4], pl[NV][4], t[NV][4];

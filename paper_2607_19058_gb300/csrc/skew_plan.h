@@ -199,6 +199,8 @@ struct StepArgs {
     double coef_plain;     // sqrt(1-beta2^t)
     uint32_t step_lo;
     uint32_t seed_lo, seed_hi;
+    const float *gscale;   // device pointer to the step's gradient scale gamma (the trainer's
+                           // global-norm clip factor), or null for gamma = 1
 };
 
 // The phases of one step: item lists (tensor, local tile / item) in device

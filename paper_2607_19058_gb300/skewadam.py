@@ -29,7 +29,7 @@ KIND_FULL, KIND_FACTORED = 0, 1
 EXPORTS = ["skew_create", "skew_destroy", "skew_state_bytes", "skew_workspace_bytes", "skew_bind", "skew_step",
            "skew_sync_status", "skew_tensor_scalars", "skew_matrix_scalars", "skew_tensor_info", "skew_num_tensors", "skew_last_error",
            "skew_profile_begin", "skew_profile_end", "skew_kernel_name", "skew_step_tensor_noalloc",
-           "skew_launches_per_step", "skew_selftest_wait_timeout", "skew_noalloc_sync_status",
+           "skew_launches_per_step", "skew_selftest_wait_timeout", "skew_noalloc_sync_status", "skew_step_scaled",
            "skew_noalloc_selftest_wait_timeout"]
 
 
@@ -84,6 +84,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
         L.skew_bind.restype = C.c_int
         L.skew_step.argtypes = [vp, i64, C.c_float, u64, vp]
         L.skew_step.restype = C.c_int
+        L.skew_step_scaled.argtypes = [vp, i64, C.c_float, u64, vp, vp]
+        L.skew_step_scaled.restype = C.c_int
         L.skew_sync_status.argtypes = [vp, vp]
         L.skew_sync_status.restype = C.c_int
         L.skew_selftest_wait_timeout.argtypes = [vp, vp]
@@ -152,6 +154,11 @@ def skew_bind(h, state_ptr: int, state_bytes: int, ws_ptr: int, ws_bytes: int, s
 
 def skew_step(h, step: int, lr: float, seed: int, stream: int) -> None:
     _check(load().skew_step(h, step, lr, seed & (2**64 - 1), stream), h)
+
+
+def skew_step_scaled(h, step: int, lr: float, seed: int, grad_scale_ptr: int, stream: int) -> None:
+    """skew_step on gamma * G, gamma read by the kernels from the device pointer (0: gamma = 1)."""
+    _check(load().skew_step_scaled(h, step, lr, seed & (2**64 - 1), grad_scale_ptr or None, stream), h)
 
 
 def skew_sync_status(h, stream: int) -> None:
@@ -301,8 +308,15 @@ class SkewAdam:
     def workspace_bytes(self) -> int:
         return skew_workspace_bytes(self.h)
 
-    def step(self, step: int, lr: float, seed: int, stream=None) -> None:
-        skew_step(self.h, step, lr, seed, self._stream(stream))
+    def step(self, step: int, lr: float, seed: int, stream=None, grad_scale=None) -> None:
+        """One step. `grad_scale`: optional one-element fp32 device tensor gamma (the trainer's
+        global gradient-norm clip factor); the step then sees gamma * G."""
+        if grad_scale is None:
+            skew_step(self.h, step, lr, seed, self._stream(stream))
+            return
+        if not (grad_scale.is_cuda and grad_scale.dtype == self.torch.float32 and grad_scale.numel() == 1):
+            raise ValueError("grad_scale must be a one-element float32 CUDA tensor")
+        skew_step_scaled(self.h, step, lr, seed, grad_scale.data_ptr(), self._stream(stream))
 
     def sync_status(self, stream=None) -> None:
         skew_sync_status(self.h, self._stream(stream))

@@ -187,7 +187,9 @@ class Harness:
     def __init__(self, wl: WL.Workload, check: Optional[Sequence[int]] = None, device="cuda",
                  grad_device: Optional[str] = None, hp_override: Optional[dict] = None,
                  misalign: Sequence[int] = (), matrices: Optional[Dict[int, Sequence[int]]] = None):
-        """`matrices[k]`, when given, limits the check of stacked tensor k to those matrices."""
+        """`matrices[k]`, when given, limits the check of stacked tensor k to those matrices.
+        `step(..., gscale=g)` steps on g * G (the trainer's global-norm clip factor), passed
+        to the GPU as a device scalar and to the oracle as its gscale."""
         self.wl = wl
         hpd = dataclasses.asdict(wl.hp)
         if hp_override:
@@ -243,9 +245,11 @@ class Harness:
             out.append(d)
         return out
 
-    def step(self, t: int, seed: int = 1234, grads_loaded: bool = False) -> Report:
+    def step(self, t: int, seed: int = 1234, grads_loaded: bool = False, gscale: Optional[float] = None) -> Report:
         if not grads_loaded:
             self.load_grads(t)
+        self.gscale = 1.0 if gscale is None else float(np.float32(gscale))
+        self.ohp.gscale = self.gscale
         torch.cuda.synchronize()
         pre = {}
         for k in self.check:   # teacher forcing: the oracle starts from the GPU's pre-step values
@@ -259,7 +263,10 @@ class Harness:
                         getattr(st, key)[:] = gs[e][key]
                 pre[k][e] = (wb[e * nm:(e + 1) * nm].copy(), gb[e * nm:(e + 1) * nm].copy(),
                              None if st.M is None else st.M.copy())
-        self.opt.step(t, self.lr, seed)
+        if gscale is None:
+            self.opt.step(t, self.lr, seed)
+        else:
+            self.opt.step(t, self.lr, seed, grad_scale=torch.tensor([gscale], dtype=torch.float32, device=self.dev))
         self.opt.sync_status()
         rep = Report()
         for k in self.check:
@@ -289,7 +296,7 @@ class Harness:
         for key in ("M", "v", "R", "C"):
             if getattr(st, key) is not None:
                 if key == "M":
-                    gd = as_f64(g)
+                    gd = self.gscale * as_f64(g)
                     b1 = float(np.float32(self.hpd["beta1"]))
                     scale = b1 * np.abs(m_prev.astype(np.float64)) + (1 - b1) * np.abs(gd)
                     err = rel_err_terms(gs[key], st.M, scale)
@@ -322,7 +329,7 @@ class Harness:
                 vhat = (st.R[i].astype(np.float64) * st.C[j].astype(np.float64) / o["rbar"]
                         if o["rbar"] > 0 else np.zeros(idx.size))
             inv = 1.0 / np.sqrt(np.maximum(vhat, eps))
-            gd = as_f64(g[idx])
+            gd = self.gscale * as_f64(g[idx])
             mterms = b1 * np.abs(m_prev[idx].astype(np.float64)) + (1 - b1) * np.abs(gd)
             return lr * o["kappa"] * coef * inv * mterms
         return fn
