@@ -20,6 +20,10 @@ post-step results are compared with the acceptance bars of the method:
     x to within ~1e-7 S, which may span several ulps of the small x. A wrong
     draw r or a wrong update is not admitted by the bound;
   * per-tensor RMS(U) and clip factor: relative error <= 1e-6.
+Every step also counts the elements that pass only through the widened readings:
+weights whose x lies within 1e-6 S but not within 1e-6 |x| of the dither's set
+(w_widened), and momenta within 1e-5 of their terms' scale but not of their value
+(m_widened); the full-size subsets assert these stay within the 1e-4 share.
 Tensors are independent, so checking a subset of a large parameter set is
 exact parity for that subset while the GPU runs the whole set. A stacked
 (E, n, m) tensor is checked as E matrices, each against its own oracle run
@@ -41,6 +45,35 @@ STATE_RTOL = 1e-5
 W_MISMATCH_FRAC = 1e-4
 X_RTOL = 1e-6
 SCALAR_RTOL = 1e-6
+# fp32 spaces its subnormals 2^-149 apart, so a state value below the normal range cannot
+# be evaluated in fp32 to 1e-5 relative: state is also accepted within a few such steps
+STATE_ATOL = 4.0 * 2.0 ** -149
+
+
+def fma_f32(a: np.ndarray, b: np.ndarray, c: np.ndarray) -> np.ndarray:
+    """fp32 fused multiply-add, correctly rounded (what fmaf / FFMA compute), emulated
+    exactly for results in fp32's normal range: a*b is exact in fp64, TwoSum gives
+    a*b + c = s + e exactly (s = fl64(a*b + c), |e| <= half an fp64 ulp of s), and
+    rounding s to fp32 equals rounding s + e unless s is itself an fp32 rounding midpoint,
+    where the sign of e decides."""
+    a = np.asarray(a, np.float32).astype(np.float64)
+    b = np.asarray(b, np.float32).astype(np.float64)
+    c = np.asarray(c, np.float32).astype(np.float64)
+    p = a * b
+    s = p + c
+    bp = s - p
+    e = (p - (s - bp)) + (c - bp)
+    r = s.astype(np.float32)
+    # an fp32 midpoint in fp64: the 29 significand bits below fp32's are 1000...0
+    mid = (s.view(np.uint64) & np.uint64((1 << 29) - 1)) == np.uint64(1 << 28)
+    fix = np.nonzero(mid & (e != 0))[0]
+    if fix.size:
+        t = r[fix]
+        below = t.astype(np.float64) < s[fix]
+        lo = np.where(below, t, np.nextafter(t, np.float32(-np.inf)))
+        hi = np.where(below, np.nextafter(t, np.float32(np.inf)), t)
+        r[fix] = np.where(e[fix] > 0, hi, lo)
+    return r
 
 
 def bits16(t: torch.Tensor) -> np.ndarray:
@@ -75,10 +108,18 @@ class Report:
     worst_thresh: float = 0.0
     clipped: int = 0
     tensors: int = 0
+    w_widened: int = 0     # weights passing only because S > |x| (reading R18)
+    m_widened: int = 0     # momenta passing only because their terms' scale > |M| (reading R17)
+    m_unexplained: int = 0  # of those, momenta that are not fma(b1, M_prev, fl(c1 g)) in fp32
+    s_floor: int = 0       # state values passing only through the subnormal floor (reading R24)
 
     def merge(self, o: "Report"):
         self.elements += o.elements
         self.w_mismatch += o.w_mismatch
+        self.w_widened += o.w_widened
+        self.m_widened += o.m_widened
+        self.m_unexplained += o.m_unexplained
+        self.s_floor += o.s_floor
         self.worst_state_rel = max(self.worst_state_rel, o.worst_state_rel)
         self.worst_scalar_rel = max(self.worst_scalar_rel, o.worst_scalar_rel)
         self.worst_thresh = max(self.worst_thresh, o.worst_thresh)
@@ -87,18 +128,27 @@ class Report:
 
 
 def rel_err(a: np.ndarray, b: np.ndarray) -> float:
-    """Max relative error of fp32 state `a` against the oracle's `b` (exact zeros must match)."""
+    """Max error of fp32 state `a` against the oracle's `b`, relative to max(|b|, the floor
+    below which fp32 state is judged in absolute terms): an element passes at STATE_RTOL
+    when it is within STATE_RTOL * |b| or within STATE_ATOL of b."""
     a = a.astype(np.float64)
     b = b.astype(np.float64)
     if not (np.isfinite(a).all() and np.isfinite(b).all()):
         return 0.0 if np.array_equal(a, b, equal_nan=True) else float("inf")
     if a.size == 0:
         return 0.0
-    d = np.abs(a - b)
-    zero = b == 0
-    if np.any(d[zero] != 0):
-        return float("inf")
-    return float((d[~zero] / np.abs(b[~zero])).max()) if (~zero).any() else 0.0
+    den = np.maximum(np.abs(b), STATE_ATOL / STATE_RTOL)
+    return float((np.abs(a - b) / den).max())
+
+
+def floor_only(a: np.ndarray, b: np.ndarray) -> int:
+    """Elements of `a` within STATE_ATOL of `b` but not within STATE_RTOL * |b| (state in
+    fp32's subnormal range)."""
+    a = a.astype(np.float64)
+    b = b.astype(np.float64)
+    fin = np.isfinite(a) & np.isfinite(b)
+    d = np.abs(a - b)[fin]
+    return int(np.count_nonzero((d > STATE_RTOL * np.abs(b[fin])) & (d <= STATE_ATOL)))
 
 
 def rel_err_terms(a: np.ndarray, b: np.ndarray, scale: np.ndarray) -> float:
@@ -113,6 +163,35 @@ def rel_err_terms(a: np.ndarray, b: np.ndarray, scale: np.ndarray) -> float:
     if np.any(d[zero] != 0):
         return float("inf")
     return float((d[~zero] / den[~zero]).max()) if (~zero).any() else 0.0
+
+
+def widened_terms(a: np.ndarray, b: np.ndarray, scale: np.ndarray, rtol: float) -> np.ndarray:
+    """Indices of the elements of `a` within rtol of `b` measured against the terms' scale
+    but not against |b|."""
+    a = a.astype(np.float64)
+    b = b.astype(np.float64)
+    d = np.abs(a - b)
+    ok = np.isfinite(a) & np.isfinite(b)
+    return np.nonzero(ok & (d > rtol * np.abs(b)) & (d <= rtol * np.maximum(np.abs(b), scale)))[0]
+
+
+def check_momentum(gpu_m: np.ndarray, ora_m: np.ndarray, m_prev: np.ndarray, g: np.ndarray, b1: float,
+                   gscale: float = 1.0):
+    """Momentum M = b1 M_prev + (1 - b1) gamma g (Algorithm 1) from the GPU against the
+    oracle's fp64 value. Returns (error relative to max(|M|, the terms' scale), the count of
+    elements passing only because their terms' scale exceeds |M| (reading R17), and how many
+    of those are not, bit for bit, fp32's fma(b1, M_prev, fl(c1 g)) with c1 = fl(1 - b1) gamma:
+    a momentum that cancels far below its terms is accepted only as that fp32 evaluation)."""
+    gd = gscale * as_f64(g)
+    scale = b1 * np.abs(m_prev.astype(np.float64)) + (1 - b1) * np.abs(gd)
+    err = rel_err_terms(gpu_m, ora_m, scale)
+    wid = widened_terms(gpu_m, ora_m, scale, STATE_RTOL)
+    if wid.size == 0:
+        return err, 0, 0
+    c1 = np.float32(np.float32(1.0 - b1) * np.float32(gscale))
+    want = fma_f32(np.full(wid.size, np.float32(b1)), m_prev[wid], c1 * as_f64(g[wid]).astype(np.float32))
+    unexplained = int(np.count_nonzero(want.view(np.uint32) != np.asarray(gpu_m, np.float32)[wid].view(np.uint32)))
+    return err, int(wid.size), unexplained
 
 
 def _bits_to_f64(b32: np.ndarray) -> np.ndarray:
@@ -131,17 +210,19 @@ def compare_weights_f32(gpu_w: np.ndarray, x: np.ndarray, w_pre: np.ndarray, wdf
         f"{where}: non-finite fp32 weights differ"
     diff = (gpu_w.view(np.uint32) != x.view(np.uint32)) & fin
     nbad = int(diff.sum())
-    worst = 0.0
+    worst, widened = 0.0, 0
     if nbad:
         t1 = w_pre[diff].astype(np.float64) * wdf
         upd = np.abs(t1 - x64[diff])
         if upd_terms is not None:
             upd = np.maximum(upd, upd_terms(np.nonzero(diff)[0]))
         S = np.abs(t1) + upd
-        rel = np.abs(g64[diff] - x64[diff]) / np.maximum(S, 1e-300)
+        dist = np.abs(g64[diff] - x64[diff])
+        rel = dist / np.maximum(S, 1e-300)
         worst = float(rel.max())
         assert worst <= X_RTOL, f"{where}: fp32 weight {worst:.3e} S from the oracle's x"
-    return 0, worst
+        widened = int(np.count_nonzero(dist > X_RTOL * np.abs(x64[diff])))
+    return 0, worst, widened
 
 
 def compare_weights(gpu_w: np.ndarray, ora_w: np.ndarray, x: np.ndarray, r: np.ndarray, w_pre: np.ndarray,
@@ -155,7 +236,7 @@ def compare_weights(gpu_w: np.ndarray, ora_w: np.ndarray, x: np.ndarray, r: np.n
     """
     diff = gpu_w != ora_w
     nbad = int(diff.sum())
-    worst = 0.0
+    worst, widened = 0.0, 0
     if nbad:
         g = gpu_w[diff].astype(np.int64)
         rr = r[diff].astype(np.int64)
@@ -178,7 +259,8 @@ def compare_weights(gpu_w: np.ndarray, ora_w: np.ndarray, x: np.ndarray, r: np.n
         k = int(np.argmax(rel))
         assert worst <= X_RTOL, (f"{where}: GPU bf16 {g[k]:#06x} is not a dithered rounding of any value within "
                                  f"{X_RTOL:g}*S of x={xo[k]!r} (S={S[k]:.3e}, distance {worst:.3e} S)")
-    return nbad, worst
+        widened = int(np.count_nonzero(dist > X_RTOL * np.abs(xo)))
+    return nbad, worst, widened
 
 
 class Harness:
@@ -186,7 +268,8 @@ class Harness:
 
     def __init__(self, wl: WL.Workload, check: Optional[Sequence[int]] = None, device="cuda",
                  grad_device: Optional[str] = None, hp_override: Optional[dict] = None,
-                 misalign: Sequence[int] = (), matrices: Optional[Dict[int, Sequence[int]]] = None):
+                 misalign: Sequence[int] = (), matrices: Optional[Dict[int, Sequence[int]]] = None,
+                 max_widened_frac: Optional[float] = None):
         """`matrices[k]`, when given, limits the check of stacked tensor k to those matrices.
         `step(..., gscale=g)` steps on g * G (the trainer's global-norm clip factor), passed
         to the GPU as a device scalar and to the oracle as its gscale."""
@@ -220,6 +303,7 @@ class Harness:
         self.ohp = O.hparams(hpd["beta1"], hpd["beta2"], hpd["eps"], hpd["clip_d"], hpd["weight_decay"],
                              annealed=hpd["policy"] == WL.POLICY_ADAFACTOR)
         self.lr = hpd["lr"]
+        self.max_widened_frac = max_widened_frac
 
     def load_grads(self, t: int):
         for k in range(len(self.wl.specs)):
@@ -275,6 +359,16 @@ class Harness:
                 rep.merge(self._check_matrix(k, e, st, pre[k][e], gws, gss[e], t, seed))
         assert rep.w_mismatch <= W_MISMATCH_FRAC * rep.elements, \
             f"{self.wl.name} step {t}: {rep.w_mismatch} of {rep.elements} weights differ"
+        print(f"parity {self.wl.name} step {t}: {rep.elements} weights, {rep.w_mismatch} one-ulp dither "
+              f"mismatches; passing only through a reading: {rep.w_widened} weights (R18), {rep.m_widened} "
+              f"momenta (R17; {rep.m_unexplained} of them not fp32's fma(b1, M_prev, fl(c1 g))), "
+              f"{rep.s_floor} state values (R24)")
+        if self.max_widened_frac is not None:
+            assert rep.w_widened <= self.max_widened_frac * rep.elements, \
+                f"{self.wl.name} step {t}: {rep.w_widened} weights pass only through reading R18"
+            assert rep.m_unexplained == 0, \
+                f"{self.wl.name} step {t}: {rep.m_unexplained} momenta pass only through reading R17 and are " \
+                f"not the fp32 evaluation of their update"
         return rep
 
     def _check_matrix(self, k, e, st, pre, gws, gs, t, seed) -> Report:
@@ -289,19 +383,18 @@ class Harness:
         wdf = 1.0 - float(np.float32(self.lr)) * lam
         terms = self._momentum_update_terms(st, o, g, m_prev, t) if st.momentum else None
         if gw.dtype == np.float32:
-            nbad, worst = compare_weights_f32(gw, o["x"], wpre, wdf, where, terms)
+            nbad, worst, wwid = compare_weights_f32(gw, o["x"], wpre, wdf, where, terms)
         else:
-            nbad, worst = compare_weights(gw, w0, o["x"], o["r"], wpre, wdf, where, terms)
-        worst_state = 0.0
+            nbad, worst, wwid = compare_weights(gw, w0, o["x"], o["r"], wpre, wdf, where, terms)
+        worst_state, mwid, munex, sfloor = 0.0, 0, 0, 0
         for key in ("M", "v", "R", "C"):
             if getattr(st, key) is not None:
                 if key == "M":
-                    gd = self.gscale * as_f64(g)
-                    b1 = float(np.float32(self.hpd["beta1"]))
-                    scale = b1 * np.abs(m_prev.astype(np.float64)) + (1 - b1) * np.abs(gd)
-                    err = rel_err_terms(gs[key], st.M, scale)
+                    err, mwid, munex = check_momentum(gs[key], st.M, m_prev, g, float(np.float32(self.hpd["beta1"])),
+                                                      self.gscale)
                 else:
                     err = rel_err(gs[key], getattr(st, key))
+                    sfloor += floor_only(gs[key], getattr(st, key))
                 assert err <= STATE_RTOL, f"{where}: state {key} rel err {err:.3g}"
                 worst_state = max(worst_state, err)
         sc = self.opt.scalars(k, matrix=e)
@@ -313,7 +406,8 @@ class Harness:
             assert err <= SCALAR_RTOL, f"{where}: {key} {sc[key]!r} vs oracle {o[key]!r}"
             se = max(se, err)
         return Report(elements=gw.size, w_mismatch=nbad, worst_state_rel=worst_state, worst_scalar_rel=se,
-                      worst_thresh=worst, clipped=int(o["kappa"] < 1.0), tensors=1)
+                      worst_thresh=worst, clipped=int(o["kappa"] < 1.0), tensors=1, w_widened=wwid, m_widened=mwid,
+                      m_unexplained=munex, s_floor=sfloor)
 
     def _momentum_update_terms(self, st, o, g, m_prev, t):
         """lr*kappa*coef/D * (b1|M_prev| + (1-b1)|g|) from the oracle's post-step state."""

@@ -152,7 +152,7 @@ def test_slice_full_size_subset():
     wl = WL.slice_()
     chk = _subset(wl, ["attn.q", "attn.k", "norm.attn", "router", "expert0.w0", "expert0.w1", "expert77.w2",
                        "expert127.w1"])
-    h = _harness(wl, check=chk)
+    h = _harness(wl, check=chk, max_widened_frac=1e-4)
     for t in (1, 2, 3):
         h.step(t)
     h.close()
@@ -162,7 +162,7 @@ def test_appb_full_size_subset():
     wl = WL.appb()
     chk = _subset(wl, ["embed", "pos", "b0.ln1.weight", "b0.attn.k", "b1.attn.o", "b1.router", "expert3.w1",
                        "expert127.w2", "ln_f.bias"])
-    h = _harness(wl, check=chk)
+    h = _harness(wl, check=chk, max_widened_frac=1e-4)
     for t in (1, 2):
         h.step(t)
     h.close()
@@ -175,7 +175,7 @@ def test_skewed_full_size_subset():
     zero_e = int(np.argmax(ranks.numpy()))          # least loaded at step 7 -> zero grads
     busy_e = int(np.argmin(ranks.numpy()))
     chk = _subset(wl, ["b1.router", "b0.attn.q", f"expert{zero_e}.w0", f"expert{busy_e}.w1", "b0.ln2.bias"])
-    h = _harness(wl, check=chk)
+    h = _harness(wl, check=chk, max_widened_frac=1e-4)
     clipped = 0
     for t in range(1, 8):
         if t in (1, 6, 7):
@@ -191,7 +191,7 @@ def test_skewed_full_size_subset():
 def test_ablation_awkward_full_size_subset():
     wl = WL.ablation()
     chk = _subset(wl, ["embed", "odd.a", "odd.b", "b1.router", "expert0.w0", "expert5.w2", "b1.ln2.weight"])
-    h = _harness(wl, check=chk)
+    h = _harness(wl, check=chk, max_widened_frac=1e-4)
     for t in (1, 2):
         h.step(t)
     h.close()
@@ -278,7 +278,7 @@ def test_stacked_appb_experts_full_size_subset():
     names = {"b1.router", "experts.w0"}
     check = [k for k, s in enumerate(wl.specs) if s.name in names]
     assert len(check) == 2
-    h = _harness(wl, check=check, matrices={check[1]: (0, 1, 77, 127)})
+    h = _harness(wl, check=check, max_widened_frac=1e-4, matrices={check[1]: (0, 1, 77, 127)})
     h.step(1, seed=3)
     h.close()
 
