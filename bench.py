@@ -22,14 +22,17 @@ Reported (one JSON line, rank 0):
                  in from pinned host memory and the weights read back each step
                  (the step run as --e2e-groups handles over runs of consecutive
                  tensors, so one group's copies overlap the others' steps);
-  cpu_baseline-- the CPU oracle (single thread) on a bounded sample;
+  cpu_baseline-- one step of the CPU oracle over the whole workload (a sample only when it
+                 would not fit the time or host-memory budget), its tensors spread over
+                 the host's cores;
   clocks      -- SM clocks and throttle reasons sampled during the timed steps.
 Multi-GPU (torchrun): every rank updates its own full parameter set (the step
 has no cross-tensor coupling, so it shards by tensor with no collective);
 scaling is weak.
 
 --impl reference times the CPU oracle (the reference arm of this benchmark) on
-the host cores instead, on bounded samples of the same workload.
+the host cores instead: each step the whole workload when --steps + --warmup of
+them fit --ref-seconds, else a sample of it; ms_per_step is the time of what ran.
 """
 import argparse
 import hashlib
@@ -60,8 +63,9 @@ def parse():
     p.add_argument("--e2e-groups", type=int, default=4, help="tensor groups of the end-to-end leg's pipeline")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--cpu-seconds", type=float, default=15.0, help="target oracle time of the CPU baseline sample")
-    p.add_argument("--ref-seconds", type=float, default=150.0, help="target total time of --impl reference")
+    p.add_argument("--cpu-seconds", type=float, default=30.0,
+                   help="oracle time budget of the CPU baseline (a full step when it fits, else a sample)")
+    p.add_argument("--ref-seconds", type=float, default=300.0, help="target total time of --impl reference")
     p.add_argument("--grad-scale", type=float, default=None,
                    help="step on gamma * G with gamma a device scalar (the trainer's global-norm clip inside the step)")
     return p.parse_args()
@@ -169,13 +173,15 @@ def byte_model(opt, n_tensors):
     return dict(N=N, N_mom=N_mom, N_full=N_full, rc=rc, step_min=step_min, kernels=kernels)
 
 
-def recorded_traffic(kernel, workload):
-    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu summary
-    (profiles/dram_traffic_appb.md, `traffic:` lines), or None when there is none or the
-    kernel source has changed since the counters were taken (its SHA-256 differs)."""
+def recorded_traffic(kernel, alg_bytes):
+    """DRAM bytes per launch of `kernel` from the committed ncu record, which is taken on
+    the 558M-parameter `small` workload (a few GB on the device; profiles/dram_traffic_small.md,
+    `traffic:` lines) and scaled to this launch by its algorithmic bytes (the kernel's
+    traffic grows with the units it processes). None when there is no record or the kernel
+    source has changed since the counters were taken (its SHA-256 differs)."""
     root = os.path.dirname(os.path.abspath(__file__))
     src = os.path.join(root, "paper_2607_19058_gb300", "csrc", "skew_kernels.cu")
-    summ = os.path.join(root, "profiles", "dram_traffic_appb.md")
+    summ = os.path.join(root, "profiles", "dram_traffic_small.md")
     try:
         with open(src, "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()
@@ -186,8 +192,8 @@ def recorded_traffic(kernel, workload):
         if not ln.startswith("traffic:"):
             continue
         kv = dict(x.split("=", 1) for x in ln[len("traffic:"):].split())
-        if kv.get("kernel") == kernel and kv.get("workload") == workload and kv.get("source_sha256") == sha:
-            return int(kv["per_launch"])
+        if kv.get("kernel") == kernel and kv.get("source_sha256") == sha and int(kv.get("alg_bytes", 0)) > 0:
+            return int(round(int(kv["per_launch"]) * alg_bytes / int(kv["alg_bytes"])))
     return None
 
 
@@ -231,6 +237,44 @@ def mem_available():
     return None
 
 
+def gpu_numa(dev_index):
+    """The NUMA node of GPU `dev_index` (sysfs, from its PCI address) and that node's CPUs;
+    read-only queries. None values where the host does not say."""
+    try:
+        out = subprocess.run(["nvidia-smi", "--query-gpu=pci.bus_id", "--format=csv,noheader", "-i", str(dev_index)],
+                             capture_output=True, text=True, timeout=30).stdout.strip()
+        bus = out.lower()
+        if bus.count(":") == 2 and len(bus.split(":")[0]) > 4:  # 00000009:01:00.0 -> 0009:01:00.0
+            bus = bus[-12:]
+        node = int(open(f"/sys/bus/pci/devices/{bus}/numa_node").read().strip())
+        cpus = None
+        if node >= 0:
+            cpus = set()
+            for part in open(f"/sys/devices/system/node/node{node}/cpulist").read().strip().split(","):
+                lo, _, hi = part.partition("-")
+                cpus.update(range(int(lo), int(hi or lo) + 1))
+        return {"gpu_pci": bus, "gpu_numa_node": node, "node_cpus": sorted(cpus) if cpus else None}
+    except Exception:
+        return {"gpu_pci": None, "gpu_numa_node": None, "node_cpus": None}
+
+
+def pages_by_node(ptr):
+    """NUMA nodes holding the pages of the mapping that contains host address `ptr`
+    (/proc/self/numa_maps), as {node: pages}; None where unavailable."""
+    try:
+        for ln in open("/proc/self/numa_maps"):
+            f = ln.split()
+            start = int(f[0], 16)
+            # numa_maps gives only starts: take the last mapping starting at or below ptr
+            if start <= ptr:
+                best = f
+            else:
+                break
+        return {int(x[1:x.index("=")]): int(x.split("=")[1]) for x in best if x.startswith("N") and "=" in x}
+    except Exception:
+        return None
+
+
 def host_info():
     """The host the CPU oracle runs on: its logical CPU count and CPU model."""
     import platform
@@ -246,30 +290,69 @@ def host_info():
     return {"nproc": os.cpu_count(), "cpu": model or platform.machine()}
 
 
-def time_oracle(wl, tids, inputs, step, lr, seed):
+def oracle_threads():
+    """Host threads for the CPU oracle: the tensors of a step are independent, and the oracle
+    is plain C called through ctypes (which releases the GIL), so a thread per core runs them
+    side by side."""
+    return max(1, os.cpu_count() or 1)
+
+
+def time_oracle(wl, tids, inputs, step, lr, seed, threads=1, states=None):
+    """Wall time of one oracle step over tensors `tids` (inputs[k] = (w bits, g bits); w is
+    updated in place), the tensors spread over `threads` host threads, largest first."""
+    import concurrent.futures as cf
     import oracle as O
     from paper_2607_19058_gb300 import workloads as WL
     hpd = wl.hp
     ohp = O.hparams(hpd.beta1, hpd.beta2, hpd.eps, hpd.clip_d, hpd.weight_decay,
                     annealed=hpd.policy == WL.POLICY_ADAFACTOR)
-    states = {k: O.TensorState(wl.specs[k].shape, wl.specs[k].tier, hpd.policy, wl.specs[k].no_decay) for k in tids}
-    t0 = time.perf_counter()
+    if states is None:
+        states = {}
     for k in tids:
+        if k not in states:
+            states[k] = O.TensorState(wl.specs[k].shape, wl.specs[k].tier, hpd.policy, wl.specs[k].no_decay)
+    O.lib()  # loaded before the threads start
+    order = sorted(tids, key=lambda k: -wl.specs[k].numel)
+
+    def one(k):
         w, g = inputs[k]
         O.tensor_step(w, g, states[k], k, ohp, step, lr, seed)
+
+    t0 = time.perf_counter()
+    if threads <= 1:
+        for k in order:
+            one(k)
+    else:
+        with cf.ThreadPoolExecutor(threads) as ex:
+            list(ex.map(one, order))
     return time.perf_counter() - t0
 
 
-def cpu_inputs(wl, tids, step=1, src=None):
+def cpu_inputs(wl, tids, step=1, src=None, threads=1):
+    """bf16 bit patterns (host numpy) of the weights and step-`step` gradients of `tids`:
+    copied from the device tensors `src`, or drawn on the host."""
+    import concurrent.futures as cf
     from paper_2607_19058_gb300 import workloads as WL
-    out = {}
-    for k in tids:
+
+    def one(k):
         if src is not None:
             w, g = src[k]
-            out[k] = (WL.bf16_bits(w).copy(), WL.bf16_bits(g).copy())
-        else:
-            out[k] = (WL.bf16_bits(WL.init_weight(wl, k, "cpu")).copy(), WL.bf16_bits(WL.grad(wl, k, step, "cpu")).copy())
-    return out
+            return k, (WL.bf16_bits(w).copy(), WL.bf16_bits(g).copy())
+        return k, (WL.bf16_bits(WL.init_weight(wl, k, "cpu")).copy(), WL.bf16_bits(WL.grad(wl, k, step, "cpu")).copy())
+
+    with cf.ThreadPoolExecutor(max(1, threads)) as ex:
+        return dict(ex.map(one, tids))
+
+
+def oracle_host_bytes(wl, tids):
+    """Host memory an oracle step over `tids` holds: bf16 weights and gradients, the fp32
+    state (its closed form) and the fp64 update of the tensors running at once (at most the
+    largest ones)."""
+    import oracle as O
+    n = sum(wl.specs[k].numel for k in tids)
+    big = sorted((wl.specs[k].numel for k in tids), reverse=True)[:oracle_threads()]
+    state = O.state_bytes([(wl.specs[k].shape, wl.specs[k].tier) for k in tids], wl.hp.policy)
+    return 4 * n + state + 8 * sum(big)
 
 
 def calibrate_oracle_rate(wl):
@@ -288,33 +371,46 @@ def calibrate_oracle_rate(wl):
     return n * m / (time.perf_counter() - t0)
 
 
+def oracle_plan(wl, budget_s, nsteps):
+    """Tensors of each oracle step and how they were chosen: the whole workload when
+    `nsteps` steps of it fit `budget_s` seconds on the host's threads and its inputs fit in
+    host memory, else a sample with the tier mix kept, sized to the budget."""
+    rate = calibrate_oracle_rate(wl) * oracle_threads() * 0.8
+    avail = mem_available()
+    full = list(range(len(wl.specs)))
+    if wl.numel / rate * nsteps <= budget_s and (avail is None or oracle_host_bytes(wl, full) < 0.7 * avail):
+        return full, wl.numel, "the whole workload"
+    tids, tot = oracle_sample_specs(wl, max(1e6, rate * budget_s / max(1, nsteps)))
+    return tids, tot, f"{len(tids)} of the {len(wl.specs)} tensors ({tot} of {wl.numel} params, tier mix kept)"
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
     if rank != 0:
         return
     from paper_2607_19058_gb300 import workloads as WL
     wl = WL.get(args.workload)
-    rate = calibrate_oracle_rate(wl)
-    per_step = max(1e6, rate * args.ref_seconds / max(1, args.steps + args.warmup))
-    tids, tot = oracle_sample_specs(wl, per_step)
-    inputs = cpu_inputs(wl, tids)
+    threads = oracle_threads()
+    tids, tot, what = oracle_plan(wl, args.ref_seconds, args.steps + args.warmup)
+    inputs = cpu_inputs(wl, tids, threads=threads)
+    states = {}
     for s in range(args.warmup):
-        time_oracle(wl, tids, inputs, s + 1, wl.hp.lr, args.seed)
-    secs = [time_oracle(wl, tids, inputs, args.warmup + s + 1, wl.hp.lr, args.seed) for s in range(args.steps)]
+        time_oracle(wl, tids, inputs, s + 1, wl.hp.lr, args.seed, threads, states)
+    secs = [time_oracle(wl, tids, inputs, args.warmup + s + 1, wl.hp.lr, args.seed, threads, states)
+            for s in range(args.steps)]
     value = tot * len(secs) / sum(secs)
-    ms_full = wl.numel / value * 1e3
-    desc = f"{len(tids)} of {len(wl.specs)} tensors ({tot} of {wl.numel} params, tier mix kept) per step"
+    ms = 1e3 * sum(secs) / len(secs)
+    desc = f"each step: {what}, on {threads} host threads (tensors spread over them)"
     out = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_full, "higher_is_better": True,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "params": wl.numel, "tensors": len(wl.specs), "policy": policy_name(wl)},
-        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": desc,
+        "config": {"workload": wl.name, "params": wl.numel, "tensors": len(wl.specs), "policy": policy_name(wl),
+                   "params_per_step": tot},
+        "cpu_baseline": {"value": value, "unit": "params/s", "cores": threads, "kind": "oracle", "sample": desc,
                          "host": host_info()},
         "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-        "note": "CPU oracle (plain fp64 C, single thread) on bounded samples of the workload; ms_per_step is the "
-                "full-workload equivalent at the sampled rate",
+        "note": "CPU oracle (plain fp64 C) on the host cores; ms_per_step is the measured time of the step it ran",
     }
     print(json.dumps(out))
 
@@ -470,10 +566,46 @@ def run_ours(args):
             step += 1
             for o in opts:
                 o.step(step, hp.lr, args.seed)
+        # pinned buffers on the GPU's own NUMA node: allocate them from that node's CPUs
+        # (pages land on the node of the thread that first touches them)
+        numa = gpu_numa(vis.split(",")[local] if vis else local)
+        prev_aff = os.sched_getaffinity(0) if hasattr(os, "sched_getaffinity") else None
+        if numa["node_cpus"] and prev_aff is not None:
+            try:
+                os.sched_setaffinity(0, set(numa["node_cpus"]) & prev_aff or prev_aff)
+            except OSError:
+                pass
         hg = torch.empty(Gbuf.numel(), dtype=torch.uint8, pin_memory=True)
         hw = torch.empty(Wbuf.numel(), dtype=torch.uint8, pin_memory=True)
         hg.copy_(Gbuf)
+        hw.copy_(Wbuf)
+        numa["pinned_pages_by_node"] = {"grads": pages_by_node(hg.data_ptr()), "weights": pages_by_node(hw.data_ptr())}
+        # the link alone: one copy each way, then both at once (4 GB or less); one untimed
+        # round first (the first copies from freshly pinned pages run slower), then the mean
+        # of three timed rounds
+        nb = min(int(Gbuf.numel()), 4 << 30)
         s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        link = {}
+        for name, dirs in (("h2d", ("in",)), ("d2h", ("out",)), ("both", ("in", "out"))):
+            ta, tb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            for rep in range(4):
+                torch.cuda.synchronize()
+                if rep == 1:
+                    ta.record(stream)
+                sts = [s_in if d == "in" else s_out for d in dirs]
+                for st_ in sts:          # both directions start together
+                    st_.wait_stream(stream)
+                for d, st_ in zip(dirs, sts):
+                    with torch.cuda.stream(st_):
+                        if d == "in":
+                            Gbuf[:nb].copy_(hg[:nb], non_blocking=True)
+                        else:
+                            hw[:nb].copy_(Wbuf[:nb], non_blocking=True)
+                for st_ in sts:
+                    stream.wait_stream(st_)
+            tb.record(stream)
+            torch.cuda.synchronize()
+            link[name + "_gbs"] = 3 * len(dirs) * nb / (ta.elapsed_time(tb) * 1e-3) / 1e9
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
@@ -505,8 +637,15 @@ def run_ours(args):
         b.record(s_out)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(a.elapsed_time(b) / args.e2e_steps, world, dev)
+        if prev_aff is not None:
+            try:
+                os.sched_setaffinity(0, prev_aff)
+            except OSError:
+                pass
         e2e = {"value": job_rate(world, bm["N"], e2e_ms), "unit": "params/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int(Gbuf.numel()), "d2h_bytes_per_step": int(Wbuf.numel()),
+               "h2d_gbs": Gbuf.numel() / (e2e_ms * 1e-3) / 1e9, "d2h_gbs": Wbuf.numel() / (e2e_ms * 1e-3) / 1e9,
+               "link_alone": link, "numa": {k: v for k, v in numa.items() if k != "node_cpus"},
                "groups": len(groups),
                "path": f"skew_step via ctypes on {len(groups)} handles over runs of consecutive tensors; every "
                        "step copies all gradients in from pinned host memory and all updated weights back to "
@@ -519,14 +658,15 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        rate = calibrate_oracle_rate(wl)
-        tids, tot = oracle_sample_specs(wl, rate * args.cpu_seconds)
-        src = {k: (W[k], G[k]) for k in tids}
-        inputs = cpu_inputs(wl, tids, src=src)
-        secs = time_oracle(wl, tids, inputs, 1, hp.lr, args.seed)
-        cpu = {"value": tot / secs, "unit": "params/s", "cores": 1, "kind": "oracle", "host": host_info(),
-               "sample": f"one step of {len(tids)} of the {len(wl.specs)} tensors ({tot} params, tier mix kept) "
-                         f"in {secs:.1f} s, single-threaded fp64 C"}
+        threads = oracle_threads()
+        tids, tot, what = oracle_plan(wl, args.cpu_seconds, 1)
+        inputs = cpu_inputs(wl, tids, src={k: (W[k], G[k]) for k in tids}, threads=threads)
+        secs = time_oracle(wl, tids, inputs, 1, hp.lr, args.seed, threads)
+        del inputs
+        cpu = {"value": tot / secs, "unit": "params/s", "cores": threads, "kind": "oracle", "host": host_info(),
+               "ms_per_step": 1e3 * secs,
+               "sample": f"one step of {what} in {secs:.1f} s, plain fp64 C, tensors spread over {threads} "
+                         "host threads"}
 
     if rank == 0:
         out = {
@@ -543,9 +683,12 @@ def run_ours(args):
                     "frac_of_8tbs": step_gbs / NOMINAL_HBM_GBS, "frac_of_measured": step_gbs / peak,
                     "peak_gbs": peak, "peak_source": peak_src},
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": recorded_traffic(dom, args.workload), "algorithmic_bytes_per_launch": dom_bytes,
+                         "frac": achieved / peak, "traffic": recorded_traffic(dom, dom_bytes),
+                         "traffic_source": "ncu DRAM bytes of one launch on the small workload, scaled by algorithmic bytes",
+                         "algorithmic_bytes_per_launch": dom_bytes,
                          "launch_ms": kmean[dom], "peak_source": peak_src},
             "kernels_ms": kmean,
+            "kernel_algorithmic_bytes": bm["kernels"],
             "step_spans": step_stats,
             "e2e": e2e,
             "cpu_baseline": cpu,

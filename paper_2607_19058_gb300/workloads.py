@@ -182,8 +182,8 @@ def adafactor() -> Workload:
 
 
 def small() -> Workload:
-    """A 573M-parameter cut of the App. B set (32 experts, a 4096^2 and a 1024x4096 backbone
-    matrix, 2 norm vectors, the router): 2.3 GB of weights + gradients, well above L2,
+    """A 558M-parameter cut of the App. B set (32 experts, a 4096^2 and a 1024x4096 backbone
+    matrix, 2 norm vectors, the router): 2.2 GB of weights + gradients, well above L2,
     for profiler captures that must stay small."""
     d = 4096
     specs = [Spec("b.q", (d, d), TIER_BACKBONE), Spec("b.k", (1024, d), TIER_BACKBONE)] + _norm("ln", d)
