@@ -63,6 +63,8 @@ def parse():
     p.add_argument("--e2e-groups", type=int, default=4, help="tensor groups of the end-to-end leg's pipeline")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-threads", type=int, default=0,
+                   help="host threads of the CPU oracle (cpu_baseline and --impl reference); 0: one per core")
     p.add_argument("--cpu-seconds", type=float, default=30.0,
                    help="oracle time budget of the CPU baseline (a full step when it fits, else a sample)")
     p.add_argument("--ref-seconds", type=float, default=300.0, help="target total time of --impl reference")
@@ -290,11 +292,14 @@ def host_info():
     return {"nproc": os.cpu_count(), "cpu": model or platform.machine()}
 
 
+_ORACLE_THREADS = None
+
+
 def oracle_threads():
     """Host threads for the CPU oracle: the tensors of a step are independent, and the oracle
     is plain C called through ctypes (which releases the GIL), so a thread per core runs them
-    side by side."""
-    return max(1, os.cpu_count() or 1)
+    side by side (--cpu-threads sets another count, e.g. 1 for a single-core baseline)."""
+    return _ORACLE_THREADS or max(1, os.cpu_count() or 1)
 
 
 def time_oracle(wl, tids, inputs, step, lr, seed, threads=1, states=None):
@@ -702,7 +707,9 @@ def run_ours(args):
 
 
 def main():
+    global _ORACLE_THREADS
     args = parse()
+    _ORACLE_THREADS = args.cpu_threads if args.cpu_threads > 0 else None
     if args.impl == "reference":
         run_reference(args)
     else:
