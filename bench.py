@@ -585,62 +585,81 @@ def run_ours(args):
         hg.copy_(Gbuf)
         hw.copy_(Wbuf)
         numa["pinned_pages_by_node"] = {"grads": pages_by_node(hg.data_ptr()), "weights": pages_by_node(hw.data_ptr())}
-        # the link alone: one copy each way, then both at once (4 GB or less); one untimed
-        # round first (the first copies from freshly pinned pages run slower), then the mean
-        # of three timed rounds
+        # the link alone: one copy each way, then both at once (4 GB or less), timed over
+        # three rounds after an untimed one; taken before the end-to-end region and again
+        # after it, since the link is shared (each host CPU serves two GPUs) and its rate
+        # can change from one minute to the next
         nb = min(int(Gbuf.numel()), 4 << 30)
         s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
-        link = {}
-        for name, dirs in (("h2d", ("in",)), ("d2h", ("out",)), ("both", ("in", "out"))):
-            ta, tb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            for rep in range(4):
+
+        def link_rates():
+            out = {}
+            for name, dirs in (("h2d", ("in",)), ("d2h", ("out",)), ("both", ("in", "out"))):
+                ta, tb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                for rep in range(4):
+                    torch.cuda.synchronize()
+                    if rep == 1:
+                        ta.record(stream)
+                    sts = [s_in if d == "in" else s_out for d in dirs]
+                    for st_ in sts:          # both directions start together
+                        st_.wait_stream(stream)
+                    for d, st_ in zip(dirs, sts):
+                        with torch.cuda.stream(st_):
+                            if d == "in":
+                                Gbuf[:nb].copy_(hg[:nb], non_blocking=True)
+                            else:
+                                hw[:nb].copy_(Wbuf[:nb], non_blocking=True)
+                    for st_ in sts:
+                        stream.wait_stream(st_)
+                tb.record(stream)
                 torch.cuda.synchronize()
-                if rep == 1:
-                    ta.record(stream)
-                sts = [s_in if d == "in" else s_out for d in dirs]
-                for st_ in sts:          # both directions start together
-                    st_.wait_stream(stream)
-                for d, st_ in zip(dirs, sts):
-                    with torch.cuda.stream(st_):
-                        if d == "in":
-                            Gbuf[:nb].copy_(hg[:nb], non_blocking=True)
-                        else:
-                            hw[:nb].copy_(Wbuf[:nb], non_blocking=True)
-                for st_ in sts:
-                    stream.wait_stream(st_)
-            tb.record(stream)
-            torch.cuda.synchronize()
-            link[name + "_gbs"] = 3 * len(dirs) * nb / (ta.elapsed_time(tb) * 1e-3) / 1e9
+                out[name + "_gbs"] = 3 * len(dirs) * nb / (ta.elapsed_time(tb) * 1e-3) / 1e9
+            return out
+
+        link = link_rates()
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         ev = lambda: torch.cuda.Event(enable_timing=False)
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(s_in)
         stepped = [None] * len(groups)
         drained = [None] * len(groups)
-        for _ in range(args.e2e_steps):
-            step += 1
-            for gi, (lo, hi) in enumerate(spans):
-                if stepped[gi] is not None:
-                    s_in.wait_event(stepped[gi])       # the group's last step has read its gradients
-                with torch.cuda.stream(s_in):
-                    Gbuf[lo:hi].copy_(hg[lo:hi], non_blocking=True)
-                loaded = ev()
-                loaded.record(s_in)
-                stream.wait_event(loaded)
-                if drained[gi] is not None:
-                    stream.wait_event(drained[gi])     # the group's last weights are back on the host
-                opts[gi].step(step, hp.lr, args.seed)
-                stepped[gi] = ev()
-                stepped[gi].record(stream)
-                s_out.wait_event(stepped[gi])
-                with torch.cuda.stream(s_out):
-                    hw[lo:hi].copy_(Wbuf[lo:hi], non_blocking=True)
-                drained[gi] = ev()
-                drained[gi].record(s_out)
+
+        def e2e_steps(k):
+            nonlocal step
+            for _ in range(k):
+                step += 1
+                for gi, (lo, hi) in enumerate(spans):
+                    if stepped[gi] is not None:
+                        s_in.wait_event(stepped[gi])       # the group's last step has read its gradients
+                    with torch.cuda.stream(s_in):
+                        Gbuf[lo:hi].copy_(hg[lo:hi], non_blocking=True)
+                    loaded = ev()
+                    loaded.record(s_in)
+                    stream.wait_event(loaded)
+                    if drained[gi] is not None:
+                        stream.wait_event(drained[gi])     # the group's last weights are back on the host
+                    opts[gi].step(step, hp.lr, args.seed)
+                    stepped[gi] = ev()
+                    stepped[gi].record(stream)
+                    s_out.wait_event(stepped[gi])
+                    with torch.cuda.stream(s_out):
+                        hw[lo:hi].copy_(Wbuf[lo:hi], non_blocking=True)
+                    drained[gi] = ev()
+                    drained[gi].record(s_out)
+
+        # untimed warm-up of the whole leg, copies included: the first device access to
+        # each page of freshly pinned host memory costs extra (about 190 ms for 2 x 12 GiB
+        # here), which a step-only warm-up leaves inside the timed region
+        e2e_steps(max(1, args.warmup))
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(s_in)
+        e2e_steps(args.e2e_steps)
         b.record(s_out)
         torch.cuda.synchronize()
+        link_after = link_rates()
         e2e_ms = max_over_ranks(a.elapsed_time(b) / args.e2e_steps, world, dev)
         if prev_aff is not None:
             try:
@@ -650,7 +669,7 @@ def run_ours(args):
         e2e = {"value": job_rate(world, bm["N"], e2e_ms), "unit": "params/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int(Gbuf.numel()), "d2h_bytes_per_step": int(Wbuf.numel()),
                "h2d_gbs": Gbuf.numel() / (e2e_ms * 1e-3) / 1e9, "d2h_gbs": Wbuf.numel() / (e2e_ms * 1e-3) / 1e9,
-               "link_alone": link, "numa": {k: v for k, v in numa.items() if k != "node_cpus"},
+               "link_alone": link, "link_alone_after": link_after, "numa": {k: v for k, v in numa.items() if k != "node_cpus"},
                "groups": len(groups),
                "path": f"skew_step via ctypes on {len(groups)} handles over runs of consecutive tensors; every "
                        "step copies all gradients in from pinned host memory and all updated weights back to "
