@@ -34,7 +34,7 @@ struct TPlan {
     int64_t n = 0, m = 0, numel = 0;
     int64_t moff = -1, voff = -1, roff = -1, coff = -1;  // floats into the state
     uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
-    uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0, fci = 0;
+    uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0, at_rows = 0, atiles = 0, fci = 0;
     uint32_t f32 = 0;         // SKEW_F_FP32: fp32 weights and gradient
     // bytes into the workspace
     size_t ws_rowp = 0, ws_colp = 0, ws_bsc = 0, ws_rsum = 0, ws_u2 = 0, ws_pp = 0, ws_rmin = 0, ws_fsum = 0, ws_fmin = 0;
@@ -114,6 +114,8 @@ static void geometry(TPlan &p, bool wg_aligned) {
     p.cr = g.cr;
     p.rt_rows = g.rt_rows;
     p.rtiles = g.rtiles;
+    p.at_rows = g.at_rows;
+    p.atiles = g.atiles;
     p.fci = g.fci;
 }
 
@@ -219,7 +221,7 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
                 for (uint32_t i = 0; i < p.nfr + p.nfc; ++i) h->itemsF.push_back(make_uint2(q, i));
             }
             if (p.rowpath) {
-                for (uint32_t i = 0; i < p.rtiles; ++i) h->itemsCR.push_back(make_uint2(q, i));
+                for (uint32_t i = 0; i < p.atiles; ++i) h->itemsCR.push_back(make_uint2(q, i));
             } else {
                 for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsB.push_back(make_uint2(q, i));
                 for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsC.push_back(make_uint2(q, i));
@@ -382,6 +384,8 @@ int skew_bind(skew_handle_t *h, void *state, size_t state_bytes, void *workspace
         T.cr = p.cr;
         T.rt_rows = p.rt_rows;
         T.rtiles = p.rtiles;
+        T.at_rows = p.at_rows;
+        T.atiles = p.atiles;
         T.fci = p.fci;
     }
     auto put = [&](size_t at, const std::vector<uint2> &v) {

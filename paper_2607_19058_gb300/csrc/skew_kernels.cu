@@ -725,7 +725,7 @@ __device__ void rowsq_tile(const StepArgs &A, const TensorDev &T, TensorScal &S,
     const L lay;
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-    const uint32_t nch = (uint32_t)min((int64_t)kRowChunks, (T.n - int64_t(tile) * T.rt_rows + T.cr - 1) / T.cr);
+    const uint32_t nch = (uint32_t)min((int64_t)(T.rt_rows / T.cr), (T.n - int64_t(tile) * T.rt_rows + T.cr - 1) / T.cr);
     if (threadIdx.x == 0) {
         for (int st = 0; st < kRowStages; ++st) mbar_init(&sm.full[st], 1);
         fence_mbar_init();
@@ -1482,13 +1482,13 @@ __device__ void apply_full_tile(const StepArgs &A, const TensorDev &T, const Ten
 struct ApplyRowSmem {
     uint4 buf[kRowStages][kRowChunkBytes / 16];  // [W rows | G rows] per slot
     uint64_t full[kRowStages];
-    float a[kRowChunks * 32];                    // row scales a_i of the tile (rt_rows <= 1024)
+    float a[kRowChunks * 32];                    // row scales a_i of the tile (at_rows <= 1024)
     float red[2 * kRowThreads / 32];
 };
 
 __device__ __forceinline__ void apply_row_issue(const TensorDev &T, uint32_t tile, uint32_t c, uint32_t ca,
                                                 ApplyRowSmem &sm, uint64_t pol) {
-    const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * ca;
+    const int64_t i0 = int64_t(tile) * T.at_rows + int64_t(c) * ca;
     const uint32_t rows = (uint32_t)min((int64_t)ca, T.n - i0);
     const uint32_t bytes = rows * (uint32_t)T.m * 2u;
     const int st = c % kRowStages;
@@ -1516,7 +1516,7 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
     const Pol sp;
     for (uint32_t c = 0; c < nch; ++c) {
         const int st = c % kRowStages;
-        const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * CA;
+        const int64_t i0 = int64_t(tile) * T.at_rows + int64_t(c) * CA;
         const int rows = (int)min((int64_t)CA, T.n - i0);
         const bool ok = mbar_wait(&sm.full[st], (c / kRowStages) & 1u);
         const uint4 *bw = sm.buf[st];
@@ -1573,8 +1573,8 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
     const L lay;
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-    const int64_t r0 = int64_t(tile) * T.rt_rows;
-    const uint32_t rows_t = (uint32_t)min((int64_t)T.rt_rows, T.n - r0);
+    const int64_t r0 = int64_t(tile) * T.at_rows;
+    const uint32_t rows_t = (uint32_t)min((int64_t)T.at_rows, T.n - r0);
     const uint32_t nch = (rows_t + CA - 1) / CA;
     if (threadIdx.x == 0) {
         for (int st = 0; st < kRowStages; ++st) mbar_init(&sm.full[st], 1);
@@ -1853,7 +1853,7 @@ __device__ void rowsq_mom_tile(const StepArgs &A, const TensorDev &T, TensorScal
 struct MomApplySmem {
     uint4 buf[kMomStages][kMomSlot16];  // [W rows | M rows] per slot
     uint64_t full[kMomStages];
-    float a[kRowChunks * 32];           // row scales a_i of the tile (rt_rows <= 1024)
+    float a[kRowChunks * 32];           // row scales a_i of the tile (at_rows <= 1024)
     float red[2 * kRowThreads / 32];
 };
 
@@ -1877,7 +1877,7 @@ __device__ void apply_rows_mom_body(const StepArgs &A, const TensorDev &T, uint3
     const Pol sp;
     for (uint32_t c = 0; c < nch; ++c) {
         const int st = c % kMomStages;
-        const int64_t i0 = int64_t(tile) * T.rt_rows + int64_t(c) * CA;
+        const int64_t i0 = int64_t(tile) * T.at_rows + int64_t(c) * CA;
         const int rows = (int)min((int64_t)CA, T.n - i0);
         const bool ok = mbar_wait(&sm.full[st], (c / kMomStages) & 1u);
         const uint4 *bw = sm.buf[st];
@@ -1934,8 +1934,8 @@ __device__ void apply_rows_mom_tile(const StepArgs &A, const TensorDev &T, const
     const L lay;
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-    const int64_t r0 = int64_t(tile) * T.rt_rows;
-    const uint32_t rows_t = (uint32_t)min((int64_t)T.rt_rows, T.n - r0);
+    const int64_t r0 = int64_t(tile) * T.at_rows;
+    const uint32_t rows_t = (uint32_t)min((int64_t)T.at_rows, T.n - r0);
     const uint32_t nch = (rows_t + T.cr - 1) / T.cr;
     if (threadIdx.x == 0) {
         for (int st = 0; st < kMomStages; ++st) mbar_init(&sm.full[st], 1);

@@ -129,7 +129,7 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     const TileGeom G = plan_geometry(kind, momentum, wg_aligned, n, m, numel);
     const bool fact = kind == kKindFactored, row = fact && G.rowpath;
     const uint32_t nA = fact && !row ? G.ntiles : 0, nR = row ? G.rtiles : 0, nF = fact ? G.nfr + G.nfc : 0;
-    const uint32_t nB = row ? 0 : G.ntiles, nC = row ? 0 : G.ntiles, nCR = row ? G.rtiles : 0;
+    const uint32_t nB = row ? 0 : G.ntiles, nC = row ? 0 : G.ntiles, nCR = row ? G.atiles : 0;
 
     // ---- scratch layout inside the fixed array --------------------------------------
     size_t off = align256(kErrOffset + 16);  // the status word comes first
@@ -206,6 +206,8 @@ extern "C" int skew_step_tensor_noalloc(void *weight, const void *grad, int32_t 
     td.cr = G.cr;
     td.rt_rows = G.rt_rows;
     td.rtiles = G.rtiles;
+    td.at_rows = G.at_rows;
+    td.atiles = G.atiles;
     td.fci = G.fci;
 
     // ---- per-step scalars, as skew_step forms them ------------------------------------

@@ -23,10 +23,14 @@ constexpr int kFinChunk = 256;  // rows / columns per finalize item
 
 // Row-tile path (phase A on whole rows, no phase B unless a clamp may bind):
 // a chunk is kRowChunkBytes of consecutive whole rows of the bf16 gradient,
-// copied to shared memory by one bulk copy; a row tile is kRowChunks chunks;
-// the CTA keeps kRowStages chunks in flight.
+// copied to shared memory by one bulk copy; a phase-A row tile is kRowChunks
+// chunks (kRowChunksWide for 4096-wide matrices of at least 2048 rows, whose
+// tiles then pay their ring ramp and column partials half as often; shorter
+// matrices keep more, smaller tiles, which measured faster); a phase-C row tile
+// is always the rows of kRowChunks chunks; the CTA keeps kRowStages chunks in flight.
 constexpr int kRowChunkBytes = 32768;
 constexpr int kRowChunks = 32;
+constexpr int kRowChunksWide = 64;
 constexpr int kRowStages = 3;
 // Momentum tensors on the row path: a chunk holds kMomGBytes of bf16 rows (G in
 // phase A, W in phase C) and the same rows of fp32 M; a row tile is kMomChunks chunks.
@@ -88,6 +92,7 @@ inline StepCoefs step_coefs(const skew_hparams_t &H, int64_t step) {
 struct TileGeom {
     uint32_t lcl = 0, strips = 1, rowtiles = 1, tile_rows = 0, ntiles = 0, nfr = 0, nfc = 0;
     uint32_t rowpath = 0, cr = 0, rt_rows = 0, rtiles = 0;
+    uint32_t at_rows = 0, atiles = 0;  // row path: phase-C row tiles (momentum tensors: the phase-A tiles)
     uint32_t fci = 0;  // row path: columns per finalize item (kFinChunk / fci threads per column)
 };
 
@@ -113,8 +118,10 @@ inline TileGeom plan_geometry(uint32_t kind, uint32_t momentum, bool wg_aligned,
         g.rowpath = (wg_aligned && (m == 512 || m == 1024 || m == 2048 || m == 4096)) ? 1u : 0u;
         if (g.rowpath) {
             g.cr = (uint32_t)((momentum ? kMomGBytes : kRowChunkBytes) / (2 * m));
-            g.rt_rows = g.cr * (momentum ? kMomChunks : kRowChunks);
+            g.rt_rows = g.cr * (momentum ? kMomChunks : m == 4096 && n >= 2048 ? kRowChunksWide : kRowChunks);
             g.rtiles = (uint32_t)((n + g.rt_rows - 1) / g.rt_rows);
+            g.at_rows = momentum ? g.rt_rows : g.cr * kRowChunks;
+            g.atiles = (uint32_t)((n + g.at_rows - 1) / g.at_rows);
             g.nfr = 0;
             // tall matrices: up to 8 threads share a column, each adding every 8th tile
             uint32_t tpc = 1;
@@ -162,9 +169,11 @@ struct TensorDev {
     uint32_t nfr, nfc;  // factored: finalize items over rows / columns
     uint32_t rowpath;   // 1: whole-row phase A (k_rowsq) and the bilinear sum of U^2
     uint32_t cr;        // row path: rows per chunk
-    uint32_t rt_rows;   // row path: rows per row tile
-    uint32_t rtiles;    // row path: row tiles
+    uint32_t rt_rows;   // row path: rows per phase-A row tile
+    uint32_t rtiles;    // row path: phase-A row tiles
     uint32_t fci;       // row path: columns per finalize item
+    uint32_t at_rows;   // row path: rows per phase-C row tile (<= 1024)
+    uint32_t atiles;    // row path: phase-C row tiles
 };
 
 // Per-tensor scalars of the current step (zeroed at the start of every step).
