@@ -292,8 +292,9 @@ const char *skew_kernel_name(int32_t k);
  * workspace; this entry point instead uses a fixed scratch array compiled into
  * the library: SKEW_NOALLOC_SCRATCH_BYTES of device memory on every GPU that
  * loads the library, held until the process exits. That is enough for one
- * 4,096-wide matrix of up to about 65,000 rows (the paper's 50,304 x 4,096
- * embedding fits; the whole-row partials take 256 bytes per row); larger
+ * 4,096-wide matrix of up to about 65,000 rows with momentum (the paper's
+ * 50,304 x 4,096 embedding fits; the whole-row partials take 256 bytes per row)
+ * and about twice that without (128 bytes per row on its 256-row tiles); larger
  * tensors are rejected with SKEW_ETOOBIG before any work is enqueued.
  *
  * Arguments: weight / grad as in skew_param_desc_t (device, bf16 or with

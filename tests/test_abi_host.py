@@ -275,6 +275,11 @@ def test_noalloc_scratch_limit_on_the_host():
         assert fits == S.SKEW_ECUDA
     big = _noalloc(rows=80000, cols=4096, tier=mom, state_bytes=4 * (80000 * 4096 + 80000 + 4096))
     assert big == S.SKEW_ETOOBIG
+    # without momentum the 256-row tiles halve the partials: about twice the rows fit
+    ex = S.TIER_EXPERT
+    if not torch.cuda.is_available():
+        assert _noalloc(rows=120000, cols=4096, tier=ex, state_bytes=4 * (120000 + 4096)) == S.SKEW_ECUDA
+    assert _noalloc(rows=140000, cols=4096, tier=ex, state_bytes=4 * (140000 + 4096)) == S.SKEW_ETOOBIG
     assert _noalloc(rows=1 << 20, cols=8192) == S.SKEW_ETOOBIG
 
 
