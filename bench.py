@@ -15,13 +15,16 @@ Reported (one JSON line, rank 0):
   hbm         -- algorithmic minimum bytes per step / step time, and its share
                  of the 8 TB/s nominal and of the measured copy bandwidth;
   roofline    -- the dominant kernel's algorithmic bytes / its event-timed
-                 duration against the measured HBM copy peak;
+                 duration against the measured HBM copy peak, and its DRAM traffic
+                 (the committed one-launch ncu record of the small workload, scaled
+                 by algorithmic bytes; null once the kernel source has changed);
   kernels_ms  -- each launch's mean event-timed duration;
   step_spans  -- median / mean / min / max of the per-step times;
   e2e         -- the same metric through the C ABI with the gradients copied
                  in from pinned host memory and the weights read back each step
                  (the step run as --e2e-groups handles over runs of consecutive
-                 tensors, so one group's copies overlap the others' steps);
+                 tensors, so one group's copies overlap the others' steps), beside
+                 the host link's own rates just before and after it;
   cpu_baseline-- one step of the CPU oracle over the whole workload (a sample only when it
                  would not fit the time or host-memory budget), its tensors spread over
                  the host's cores;
