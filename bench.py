@@ -178,13 +178,13 @@ def byte_model(opt, n_tensors):
     return dict(N=N, N_mom=N_mom, N_full=N_full, rc=rc, step_min=step_min, kernels=kernels)
 
 
-def recorded_traffic(kernel, alg_bytes):
+def recorded_traffic(kernel, alg_bytes, root=None):
     """DRAM bytes per launch of `kernel` from the committed ncu record, which is taken on
     the 558M-parameter `small` workload (a few GB on the device; profiles/dram_traffic_small.md,
     `traffic:` lines) and scaled to this launch by its algorithmic bytes (the kernel's
     traffic grows with the units it processes). None when there is no record or the kernel
     source has changed since the counters were taken (its SHA-256 differs)."""
-    root = os.path.dirname(os.path.abspath(__file__))
+    root = root or os.path.dirname(os.path.abspath(__file__))
     src = os.path.join(root, "paper_2607_19058_gb300", "csrc", "skew_kernels.cu")
     summ = os.path.join(root, "profiles", "dram_traffic_small.md")
     try:
@@ -662,6 +662,16 @@ def run_ours(args):
         e2e_steps(args.e2e_steps)
         b.record(s_out)
         torch.cuda.synchronize()
+        # integrity of the leg: each group's first and last 16 MiB of updated weights in
+        # host memory equal the device's, and its gradients on the device equal the host's
+        chk = 16 << 20
+        w_ok = g_ok = True
+        checked = 0
+        for lo, hi in spans:
+            for a0, a1 in ((lo, min(hi, lo + chk)), (max(lo, hi - chk), hi)):
+                w_ok &= bool(torch.equal(hw[a0:a1].to(dev), Wbuf[a0:a1]))
+                g_ok &= bool(torch.equal(hg[a0:a1].to(dev), Gbuf[a0:a1]))
+                checked += 2 * (a1 - a0)
         link_after = link_rates()
         e2e_ms = max_over_ranks(a.elapsed_time(b) / args.e2e_steps, world, dev)
         if prev_aff is not None:
@@ -672,6 +682,7 @@ def run_ours(args):
         e2e = {"value": job_rate(world, bm["N"], e2e_ms), "unit": "params/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int(Gbuf.numel()), "d2h_bytes_per_step": int(Wbuf.numel()),
                "h2d_gbs": Gbuf.numel() / (e2e_ms * 1e-3) / 1e9, "d2h_gbs": Wbuf.numel() / (e2e_ms * 1e-3) / 1e9,
+               "verified": {"weights_back_equal": w_ok, "grads_in_equal": g_ok, "bytes_checked": checked},
                "link_alone": link, "link_alone_after": link_after, "numa": {k: v for k, v in numa.items() if k != "node_cpus"},
                "groups": len(groups),
                "path": f"skew_step via ctypes on {len(groups)} handles over runs of consecutive tensors; every "
