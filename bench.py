@@ -62,8 +62,8 @@ def parse():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="appb", help="shape set (appb = the paper's 6.78B App. B shapes)")
     p.add_argument("--seed", type=int, default=20260207)
-    p.add_argument("--e2e-steps", type=int, default=6)
-    p.add_argument("--e2e-groups", type=int, default=4, help="tensor groups of the end-to-end leg's pipeline")
+    p.add_argument("--e2e-steps", type=int, default=8)
+    p.add_argument("--e2e-groups", type=int, default=8, help="tensor groups of the end-to-end leg's pipeline")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-threads", type=int, default=0,
