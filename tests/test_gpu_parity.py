@@ -363,3 +363,36 @@ def test_momentum_row_path_fallbacks():
             h.G[5][1].zero_()
         h.step(t, seed=9, grads_loaded=True)
     h.close()
+
+
+def _wide_tile_workload():
+    """Momentum-free 4096-wide matrices of at least 2048 rows, whose phase-A tiles are 256
+    rows (phase C keeps 128): ragged last tiles of 1 row, of 63 whole chunks, and of 63
+    chunks and a 2-row chunk, a stack of two such matrices, and a 2047-row matrix (the
+    largest that keeps 128-row phase-A tiles) beside them."""
+    E = WL.TIER_EXPERT
+    specs = [WL.Spec("e2049x4096", (2049, 4096), E, expert=0), WL.Spec("e2300x4096", (2300, 4096), E, expert=1),
+             WL.Spec("e2302x4096", (2302, 4096), E, expert=2), WL.Spec("s2x2050x4096", (2, 2050, 4096), E),
+             WL.Spec("e2047x4096", (2047, 4096), E, expert=3)]
+    return WL.Workload("wide", specs, WL.HP(), "normal", steps=3)
+
+
+def test_wide_phase_a_tiles_ragged():
+    h = _harness(_wide_tile_workload())
+    assert all(h.opt.info(k).rowpath == 1 for k in range(len(h.wl.specs)))
+    for t in range(1, 4):
+        h.step(t, seed=7 * t)
+    h.close()
+
+
+def test_wide_phase_a_tiles_with_grad_scale_and_clamp():
+    """The same shapes under the trainer's clip factor, and with eps = 1e-8 (App. A), where
+    the clamp binds and the tensors take phase B."""
+    h = _harness(_wide_tile_workload())
+    for t, g in ((1, 0.37), (2, 1.0), (3, 0.8)):
+        h.step(t, seed=3 * t, gscale=g)
+    h.close()
+    h = _harness(_wide_tile_workload(), hp_override=dict(eps=1e-8, lr=3e-4, weight_decay=0.05))
+    for t in (1, 2):
+        h.step(t, seed=19 * t)
+    h.close()
