@@ -15,6 +15,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
+#include <algorithm>
 #include <cstring>
 #include <new>
 #include <string>
@@ -227,6 +228,21 @@ int skew_create(const skew_param_desc_t *params, int32_t n_params, const skew_hp
                 for (uint32_t i = 0; i < p.ntiles; ++i) h->itemsC.push_back(make_uint2(q, i));
             }
         }
+        // the last phase-C row tiles of momentum-free matrices run as two half tiles each
+        // (tiles of momentum matrices and tile indices past the mask keep whole tiles)
+        std::vector<uint2> tail;
+        const size_t ncr = h->itemsCR.size(), nsplit = std::min<size_t>(ncr, kApplyTailSplit);
+        for (size_t k = ncr - nsplit; k < ncr; ++k) {
+            const uint2 it = h->itemsCR[k];
+            if (!h->t[it.x].momentum && it.y <= kTileMask) {
+                tail.push_back(make_uint2(it.x, it.y | kHalfTile));
+                tail.push_back(make_uint2(it.x, it.y | kHalfTile | kSecondHalf));
+            } else {
+                tail.push_back(it);
+            }
+        }
+        h->itemsCR.resize(ncr - nsplit);
+        h->itemsCR.insert(h->itemsCR.end(), tail.begin(), tail.end());
     } catch (...) {
         delete h;
         return fail(nullptr, SKEW_ENOMEM, "out of host memory");

@@ -1486,9 +1486,11 @@ struct ApplyRowSmem {
     float red[2 * kRowThreads / 32];
 };
 
-__device__ __forceinline__ void apply_row_issue(const TensorDev &T, uint32_t tile, uint32_t c, uint32_t ca,
+// Chunk c of the phase-C tile (or half tile) whose first row is r0. A half tile is 16 of
+// the phase-A chunks' rows, i.e. whole phase-C chunks, so only the matrix's end cuts one.
+__device__ __forceinline__ void apply_row_issue(const TensorDev &T, int64_t r0, uint32_t c, uint32_t ca,
                                                 ApplyRowSmem &sm, uint64_t pol) {
-    const int64_t i0 = int64_t(tile) * T.at_rows + int64_t(c) * ca;
+    const int64_t i0 = r0 + int64_t(c) * ca;
     const uint32_t rows = (uint32_t)min((int64_t)ca, T.n - i0);
     const uint32_t bytes = rows * (uint32_t)T.m * 2u;
     const int st = c % kRowStages;
@@ -1499,7 +1501,7 @@ __device__ __forceinline__ void apply_row_issue(const TensorDev &T, uint32_t til
 
 // CA = 1024 / V rows per chunk (16 KB of W, 16 KB of G), KA = CA / RPP rows per thread.
 template <int TPB, int V, bool FAST>
-__device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t tile,
+__device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, int64_t r0,
                                 const float (&b)[RowLayout<TPB, V>::NV][8], float coefC, ApplyRowSmem &sm,
                                 uint32_t nch, uint64_t pol) {
     using L = RowLayout<TPB, V>;
@@ -1516,7 +1518,7 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
     const Pol sp;
     for (uint32_t c = 0; c < nch; ++c) {
         const int st = c % kRowStages;
-        const int64_t i0 = int64_t(tile) * T.at_rows + int64_t(c) * CA;
+        const int64_t i0 = r0 + int64_t(c) * CA;
         const int rows = (int)min((int64_t)CA, T.n - i0);
         const bool ok = mbar_wait(&sm.full[st], (c / kRowStages) & 1u);
         const uint4 *bw = sm.buf[st];
@@ -1559,13 +1561,13 @@ __device__ void apply_rows_body(const StepArgs &A, const TensorDev &T, uint32_t 
         }
         if (tid == 0 && c + kRowStages < nch) {
             fence_proxy_async_smem();
-            apply_row_issue(T, tile, c + kRowStages, CA, sm, pol);
+            apply_row_issue(T, r0, c + kRowStages, CA, sm, pol);
         }
     }
 }
 
 template <int TPB, int V>
-__device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t tile,
+__device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const TensorScal &S, uint32_t item,
                                 ApplyRowSmem &sm) {
     using L = RowLayout<TPB, V>;
     constexpr int NV = L::NV;
@@ -1573,8 +1575,11 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
     const L lay;
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-    const int64_t r0 = int64_t(tile) * T.at_rows;
-    const uint32_t rows_t = (uint32_t)min((int64_t)T.at_rows, T.n - r0);
+    // a whole tile, or one half of it (the step's last tiles run as halves)
+    const uint32_t trows = (item & kHalfTile) ? T.at_rows / 2 : T.at_rows;
+    const int64_t r0 = int64_t(item & kTileMask) * T.at_rows + ((item & kSecondHalf) ? trows : 0);
+    if (r0 >= T.n) return;  // the second half of a matrix's short last tile
+    const uint32_t rows_t = (uint32_t)min((int64_t)trows, T.n - r0);
     const uint32_t nch = (rows_t + CA - 1) / CA;
     if (threadIdx.x == 0) {
         for (int st = 0; st < kRowStages; ++st) mbar_init(&sm.full[st], 1);
@@ -1582,7 +1587,7 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
     }
     __syncthreads();
     if (threadIdx.x == 0)
-        for (uint32_t c = 0; c < nch && c < (uint32_t)kRowStages; ++c) apply_row_issue(T, tile, c, CA, sm, pol);
+        for (uint32_t c = 0; c < nch && c < (uint32_t)kRowStages; ++c) apply_row_issue(T, r0, c, CA, sm, pol);
     // row scales of the tile, column scales of this thread's columns, and the clamp test
     const float rbar_s = __ldcg(&S.rbar_s);
     const int rbar_e = __ldcg(&S.rbar_e);
@@ -1621,9 +1626,9 @@ __device__ void apply_rows_tile(const StepArgs &A, const TensorDev &T, const Ten
     }
     const float coefC = __ldcg(&S.coefC);
     if (ma * mb <= A.ce)
-        apply_rows_body<TPB, V, true>(A, T, tile, b, coefC, sm, nch, pol);
+        apply_rows_body<TPB, V, true>(A, T, r0, b, coefC, sm, nch, pol);
     else
-        apply_rows_body<TPB, V, false>(A, T, tile, b, coefC, sm, nch, pol);
+        apply_rows_body<TPB, V, false>(A, T, r0, b, coefC, sm, nch, pol);
 }
 
 // ---------------------------------------------------------------------------

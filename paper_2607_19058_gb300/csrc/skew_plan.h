@@ -34,6 +34,12 @@ constexpr int kRowChunksWide = 64;
 constexpr int kRowStages = 3;
 // Momentum tensors on the row path: a chunk holds kMomGBytes of bf16 rows (G in
 // phase A, W in phase C) and the same rows of fp32 M; a row tile is kMomChunks chunks.
+// Phase C on the row path: the last kApplyTailSplit tiles of a step (two waves of the
+// kernel's two CTAs per SM on GB300's 152 SMs) run as two half tiles each, so that the
+// launch's last wave ends sooner. An item's tile field then carries kHalfTile, plus
+// kSecondHalf for the second half (results do not depend on the split).
+constexpr uint32_t kApplyTailSplit = 2u * 2u * 152u;
+constexpr uint32_t kHalfTile = 1u << 31, kSecondHalf = 1u << 30, kTileMask = kSecondHalf - 1u;
 constexpr int kMomGBytes = 16384;
 constexpr int kMomChunks = 64;
 
