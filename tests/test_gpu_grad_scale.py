@@ -120,3 +120,22 @@ def test_grad_scale_is_not_a_learning_rate():
     assert int((d_gamma > 0).sum()) <= 1e-4 * n and int(d_gamma.max()) <= 1
     # a learning rate scaled by gamma shrinks every update instead
     assert int((d_lr > 0).sum()) > 0.5 * n
+
+
+def test_grad_scale_fp32_tensors():
+    """fp32 router and LayerNorm vectors (the paper's precision, App. A) beside bf16 matrices,
+    with gamma changing from step to step."""
+    h = _harness(WL.toy_fp32())
+    for t, g in ((1, 0.37), (2, 0.9), (3, 1.0), (4, 0.5)):
+        h.step(t, seed=13 * t, gscale=g)
+    h.close()
+
+
+def test_grad_scale_adafactor_comparator():
+    """The Adafactor comparator's annealed beta2_t with gamma: every increment (1 - beta2_t)
+    gamma^2 g^2, on the strip path (toy) and the whole-row path."""
+    for wl in (WL.toy(), _mixed_workload()):
+        h = _harness(wl, hp_override=dict(policy=WL.POLICY_ADAFACTOR))
+        for t, g in ((1, 0.6), (2, 0.37), (3, 1.0)):
+            h.step(t, seed=17 * t, gscale=g)
+        h.close()
